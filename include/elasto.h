@@ -1,0 +1,175 @@
+/*
+ * elasto.h -- C-ABI of libelasto: the runtime forward pass of one Descendant
+ * Network (DN) of an elastic ViT or ResNet-50, chosen at run time from one
+ * shared set of weights (Elastoformer, Section 4.3 "Elastic Neural Network").
+ *
+ * A DN ("mode") keeps, per layer, a subset of attention heads and of MLP
+ * hidden channels (ViT; Eq. 4 and Eq. 6 with structured 0/1 masks), or per
+ * bottleneck block subsets of the two inner conv widths (ResNet-50; Eq. 7).
+ * Masking whole rows/columns to zero is computed as deleting them: the library
+ * gathers each mode's kept rows/columns into contiguous packed weights once,
+ * at create time, so switching modes at run time is a pointer swap with no
+ * weight copy (the paper measures its switch cost in Section 6.2).
+ *
+ * Conventions common to every call:
+ *  - Every call returns an elasto_status; on failure a thread-local message is
+ *    available from elasto_last_error().
+ *  - Pointers named *_host are host memory; all others named device are CUDA
+ *    device memory of the current device. The library never keeps a caller
+ *    pointer past the call that received it.
+ *  - Streams are cudaStream_t passed as void* (NULL = legacy default stream).
+ *  - Asynchronous CUDA faults surface at the caller's next synchronisation,
+ *    and at the next library call as ELASTO_ERR_CUDA.
+ *  - A handle is not thread-safe: the caller serialises calls on one handle.
+ */
+#ifndef ELASTO_H
+#define ELASTO_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct elasto_s* elasto_t; /* opaque, owned by the library */
+
+typedef enum {
+  ELASTO_OK = 0,
+  ELASTO_ERR_INVALID_ARG = -1, /* null pointer, bad size, bad descriptor */
+  ELASTO_ERR_BAD_TABLE = -2,   /* kept-index table not sorted/unique/in range */
+  ELASTO_ERR_BAD_MODE = -3,    /* mode index out of range */
+  ELASTO_ERR_OOM = -4,         /* device allocation failed */
+  ELASTO_ERR_CUDA = -5,        /* CUDA runtime/driver error */
+  ELASTO_ERR_UNSUPPORTED = -6, /* shape or device the kernels do not support */
+  ELASTO_ERR_TIMEOUT = -7      /* a device-side wait gave up (status word) */
+} elasto_status;
+
+enum { ELASTO_ARCH_VIT = 1, ELASTO_ARCH_RESNET50 = 2 };
+enum { ELASTO_F32 = 0, ELASTO_BF16 = 1 };
+
+/* Model description.
+ * ViT (Section 4.1, 5.2): img_h = img_w, patch P divides img_h, n = (img_h/P)^2 + 1
+ *   tokens, dim d, heads h with d/h = 64, mlp d_ff, layers L, classes C.
+ * ResNet-50 v1.5: img_c = 3, classes C; patch/dim/heads/mlp/layers ignored
+ *   (bottlenecks [3,4,6,3], widths 64..512 are fixed).
+ * weight_dtype: storage type of the weights AND of the images given to
+ *   forward (ELASTO_F32 or ELASTO_BF16). Weights are stored on the device as
+ *   bf16 (fp32 inputs are rounded to nearest even); biases, LayerNorm
+ *   parameters, position embeddings and the classifier stay fp32.
+ * max_batch: largest batch forward accepts; sizes the activation workspace. */
+typedef struct {
+  int arch;
+  int img_h, img_w, img_c;
+  int patch, dim, heads, mlp, layers, classes;
+  int weight_dtype;
+  int max_batch;
+} elasto_model_desc;
+
+/* Weights: host pointers to the canonical tensors, PyTorch layouts, each of
+ * weight_dtype, in this fixed order.
+ * ViT (4 + 12 L + 4 tensors):
+ *   patch_w [d,C,P,P], patch_b [d], cls [d], pos [n,d],
+ *   per layer: ln1_w [d], ln1_b [d], qkv_w [3d,d], qkv_b [3d], proj_w [d,d],
+ *              proj_b [d], ln2_w [d], ln2_b [d], fc1_w [f,d], fc1_b [f],
+ *              fc2_w [d,f], fc2_b [d],
+ *   norm_w [d], norm_b [d], head_w [C,d], head_b [C].
+ *   qkv_w rows: blocks q | k | v of d rows each, head-major inside a block.
+ * ResNet-50 (5 + 15 per block + 5 per projection + 2 = 267 tensors):
+ *   stem_w [64,3,7,7], stem BN gamma, beta, mean, var [64];
+ *   per block: conv1_w [w,cin,1,1], bn1 x4, conv2_w [w,w,3,3], bn2 x4,
+ *              conv3_w [4w,w,1,1], bn3 x4, and on the first block of each
+ *              stage down_w [4w,cin,1,1], down BN x4;
+ *   fc_w [C,2048], fc_b [C]. BN eps = 1e-5, LayerNorm eps = 1e-6. */
+typedef struct {
+  const void* const* tensors;
+  int n_tensors;
+} elasto_weights;
+
+/* One mode's kept-index tables: int32, strictly increasing, in range.
+ * ViT: heads_kept is the concatenation over layers of each layer's kept head
+ *   indices (n_heads_kept[l] entries for layer l, 0 <= n <= h); mlp_kept
+ *   likewise for MLP hidden channels (0 <= n_mlp_kept[l] <= d_ff).
+ * ResNet-50: conv_kept_a / conv_kept_b concatenate, per block, the kept
+ *   channels after conv1 (S_a) and after conv2 (S_b), 1 <= n <= width.
+ * Unused members may be NULL. */
+typedef struct {
+  const int32_t* heads_kept;
+  const int32_t* n_heads_kept;
+  const int32_t* mlp_kept;
+  const int32_t* n_mlp_kept;
+  const int32_t* conv_kept_a;
+  const int32_t* n_conv_a;
+  const int32_t* conv_kept_b;
+  const int32_t* n_conv_b;
+} elasto_mode_tables;
+
+/* Build an elastic model on the current device: validates descriptor and
+ * tables, copies the weights to one library-owned device arena, packs every
+ * mode's kept rows/columns (Eq. 4, 6, 7 as deletion; "pruning metadata" of
+ * Section 4.1-4.2) and allocates the activation workspace for max_batch.
+ * Synchronous. Mode 0 is current afterwards. The caller may free all inputs
+ * when this returns. Errors: INVALID_ARG, BAD_TABLE, OOM, CUDA, UNSUPPORTED. */
+elasto_status elasto_create(const elasto_model_desc* desc, const elasto_weights* weights,
+                            const elasto_mode_tables* modes, int n_modes, elasto_t* out);
+
+/* Select the DN used by forwards enqueued after this call (Section 4.4: the
+ * runtime picks one DN). Host-only, O(1), no device work, no allocation;
+ * forwards already enqueued keep the mode they were enqueued with.
+ * Errors: INVALID_ARG (null handle), BAD_MODE. */
+elasto_status elasto_set_mode(elasto_t h, int mode);
+elasto_status elasto_get_mode(elasto_t h, int* mode);
+
+/* Enqueue the current mode's forward pass on `stream`:
+ *   images_device: [batch, img_h, img_w, img_c] NHWC of weight_dtype, device;
+ *   logits_device: [batch, classes] fp32, device, written.
+ * 1 <= batch <= max_batch. Asynchronous; never synchronises. Buffers are
+ * caller-owned. Concurrent forwards on one handle share its workspace and
+ * must be ordered on one stream. Errors: INVALID_ARG, CUDA. */
+elasto_status elasto_forward(elasto_t h, void* stream, const void* images_device, int batch,
+                             float* logits_device);
+
+/* The same forward from host memory: copies images_host to a library-owned
+ * device buffer, runs the forward, copies the logits back to logits_host and
+ * synchronises `stream` before returning (pinned host memory makes the copies
+ * asynchronous with respect to the host until that point). */
+elasto_status elasto_forward_host(elasto_t h, void* stream, const void* images_host, int batch,
+                                  float* logits_host);
+
+/* Synchronise `stream`, then read and clear the handle's device status word
+ * (kernels record ELASTO_ERR_TIMEOUT there instead of hanging). Returns the
+ * recorded status or ELASTO_OK. */
+elasto_status elasto_sync_status(elasto_t h, void* stream);
+
+/* Release everything the handle owns (synchronises the device first). */
+elasto_status elasto_destroy(elasto_t h);
+
+/* Message of the last failing call on this thread ("" if none). */
+const char* elasto_last_error(void);
+
+/* Introspection: ELASTO_Q_* values. `mode` is used where it applies. */
+enum {
+  ELASTO_Q_N_MODES = 0,
+  ELASTO_Q_PACKED_BYTES = 1,     /* device bytes of one mode's packed weights */
+  ELASTO_Q_SHARED_BYTES = 2,     /* device bytes of mode-independent weights */
+  ELASTO_Q_WORKSPACE_BYTES = 3,  /* activation workspace for max_batch */
+  ELASTO_Q_ARENA_BYTES = 4,      /* total device bytes owned by the handle */
+  ELASTO_Q_MODE_MACS = 5,        /* multiply-accumulates per image of the mode */
+  ELASTO_Q_LAUNCHES = 6          /* kernels one forward of the mode launches */
+};
+elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value);
+
+/* Test hook: copy one packed buffer of (mode, layer) to host_dst (bytes must
+ * equal its size). ViT `which`: 0 qkv_w bf16 [3w,d], 1 qkv_b fp32 [3w],
+ * 2 proj_w bf16 [d,w], 3 fc1_w bf16 [f,d], 4 fc1_b fp32 [f], 5 fc2_w bf16 [d,f]
+ * (w = 64 x kept heads, f = kept channels). ResNet-50 (layer = block):
+ * 0 conv1 bf16 [|S_a|, cin], 1 bias1 fp32, 2 conv2 bf16 [|S_b|, 3, 3, |S_a|],
+ * 3 bias2 fp32, 4 conv3 bf16 [4w, |S_b|], 5 bias3 fp32 (BN folded).
+ * Synchronous. Errors: INVALID_ARG, BAD_MODE. */
+elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int which, void* host_dst,
+                                         size_t bytes);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ELASTO_H */

@@ -1,0 +1,60 @@
+/*
+ * elasto_ops.h -- stateless kernel-level entry points of libelasto. Each is
+ * one step of the DN forward (Section 4.1, Eq. 2-7) that elasto_forward
+ * composes; they exist so that every kernel can be checked on its own
+ * against the fp64 definition of that step.
+ *
+ * All pointers are CUDA device memory of the current device, 16-byte aligned,
+ * row-major, caller-owned. Calls are asynchronous on `stream` (void* =
+ * cudaStream_t). `status_device` (nullable) is an int the kernels set to
+ * ELASTO_ERR_TIMEOUT if one of their bounded device-side waits gives up.
+ * Errors: ELASTO_ERR_INVALID_ARG for null pointers, non-positive or
+ * unsupported sizes; ELASTO_ERR_CUDA for launch failures.
+ */
+#ifndef ELASTO_OPS_H
+#define ELASTO_OPS_H
+
+#include "elasto.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Epilogues fused into the tensor-core GEMM (acc = A W^T in fp32). */
+typedef enum {
+  ELASTO_EPI_BIAS_BF16 = 0,       /* out bf16 = acc + bias                  (QKV, Eq. 2) */
+  ELASTO_EPI_BIAS_GELU_BF16 = 1,  /* out bf16 = GELU(acc + bias)            (FC1, Eq. 5) */
+  ELASTO_EPI_BIAS_RESID_F32 = 2,  /* out fp32 += acc + bias                 (proj, FC2: residual) */
+  ELASTO_EPI_BIAS_F32 = 3,        /* out fp32 = acc + bias */
+  ELASTO_EPI_BIAS_RELU_BF16 = 4,  /* out bf16 = ReLU(acc + bias)            (conv + folded BN) */
+  ELASTO_EPI_BIAS_RESID_RELU_BF16 = 5 /* out bf16 = ReLU(acc + bias + resid) (block output) */
+} elasto_epilogue;
+
+/* out[M,N] = epilogue(A[M,K] W[N,K]^T): A, W bf16 (K contiguous); bias fp32
+ * [N] or NULL (= 0); resid bf16 [M,N] only for ..._RESID_RELU_BF16. Output
+ * row stride is N. Requires K % 8 == 0, N % 2 == 0, M, N, K >= 1 (K may be 0:
+ * then acc = 0). tcgen05 MMA (M = 128 tiles), TMA-fed, persistent grid. */
+elasto_status elasto_op_gemm(void* stream, const void* A, const void* W, const float* bias, void* out,
+                             const void* resid, int M, int N, int K, int epilogue, int* status_device);
+
+/* y bf16 [rows, d] = LayerNorm(x fp32 [rows, d]) * gamma + beta, eps = 1e-6,
+ * biased variance, statistics in fp32 (one warp per row). d % 64 == 0,
+ * d <= 4096. */
+elasto_status elasto_op_layernorm(void* stream, const float* x, const float* gamma, const float* beta,
+                                  void* y, int rows, int d);
+
+/* y fp32 [rows, cols] = softmax over each row of x fp32 [rows, cols]
+ * (exp(x - max) / sum, one warp per row, warp-shuffle reductions). */
+elasto_status elasto_op_softmax(void* stream, const float* x, float* y, int rows, int cols);
+
+/* Multi-head attention over the kept heads (Eq. 3), all heads of width 64:
+ * qkv bf16 [batch, n, 3, heads, 64] (q | k | v blocks, head-major, as the
+ * QKV GEMM writes them) -> out bf16 [batch, n, heads * 64] (heads
+ * concatenated in order, Eq. 2). Scale 1/8. 1 <= n <= 256. */
+elasto_status elasto_op_attention(void* stream, const void* qkv, void* out, int batch, int n, int heads,
+                                  int* status_device);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* ELASTO_OPS_H */

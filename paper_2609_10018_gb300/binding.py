@@ -1,0 +1,301 @@
+"""ctypes binding to libelasto.so (include/elasto.h, include/elasto_ops.h).
+
+Argument marshalling only: every step of the forward pass runs in the CUDA
+library. Functions keep the C names; `ElasticModel` is a small owner of one
+handle. Device buffers are passed as integer addresses (e.g. a torch CUDA
+tensor's data_ptr()), streams as integer cudaStream_t handles (e.g.
+torch.cuda.current_stream().cuda_stream). There is no CPU fallback: if the
+library is missing this module raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Dict, List, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libelasto.so")
+
+ARCH_VIT, ARCH_RESNET50 = 1, 2
+F32, BF16 = 0, 1
+OK, ERR_INVALID_ARG, ERR_BAD_TABLE, ERR_BAD_MODE, ERR_OOM, ERR_CUDA, ERR_UNSUPPORTED, ERR_TIMEOUT = (
+    0, -1, -2, -3, -4, -5, -6, -7)
+Q_N_MODES, Q_PACKED_BYTES, Q_SHARED_BYTES, Q_WORKSPACE_BYTES, Q_ARENA_BYTES, Q_MODE_MACS, Q_LAUNCHES = range(7)
+EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_BIAS_RESID_F32, EPI_BIAS_F32, EPI_BIAS_RELU_BF16, EPI_BIAS_RESID_RELU_BF16 = range(6)
+
+c_int, c_void_p, c_size_t, c_int64 = ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int64
+P_i32 = ctypes.POINTER(ctypes.c_int32)
+
+
+class ModelDesc(ctypes.Structure):
+    _fields_ = [("arch", c_int), ("img_h", c_int), ("img_w", c_int), ("img_c", c_int), ("patch", c_int),
+                ("dim", c_int), ("heads", c_int), ("mlp", c_int), ("layers", c_int), ("classes", c_int),
+                ("weight_dtype", c_int), ("max_batch", c_int)]
+
+
+class Weights(ctypes.Structure):
+    _fields_ = [("tensors", ctypes.POINTER(c_void_p)), ("n_tensors", c_int)]
+
+
+class ModeTables(ctypes.Structure):
+    _fields_ = [("heads_kept", P_i32), ("n_heads_kept", P_i32), ("mlp_kept", P_i32), ("n_mlp_kept", P_i32),
+                ("conv_kept_a", P_i32), ("n_conv_a", P_i32), ("conv_kept_b", P_i32), ("n_conv_b", P_i32)]
+
+
+class ElastoError(RuntimeError):
+    def __init__(self, status: int, where: str, msg: str):
+        super().__init__(f"{where} failed with status {status}: {msg}")
+        self.status = status
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load libelasto.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2609_10018_gb300.build.build()")
+    L = ctypes.CDLL(LIB_PATH)
+    sig = {
+        "elasto_create": [ctypes.POINTER(ModelDesc), ctypes.POINTER(Weights), ctypes.POINTER(ModeTables), c_int,
+                          ctypes.POINTER(c_void_p)],
+        "elasto_set_mode": [c_void_p, c_int],
+        "elasto_get_mode": [c_void_p, ctypes.POINTER(c_int)],
+        "elasto_forward": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
+        "elasto_forward_host": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
+        "elasto_sync_status": [c_void_p, c_void_p],
+        "elasto_destroy": [c_void_p],
+        "elasto_query": [c_void_p, c_int, c_int, ctypes.POINTER(c_int64)],
+        "elasto_debug_export_packed": [c_void_p, c_int, c_int, c_int, c_void_p, c_size_t],
+        "elasto_op_gemm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
+                           c_void_p],
+        "elasto_op_layernorm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int],
+        "elasto_op_softmax": [c_void_p, c_void_p, c_void_p, c_int, c_int],
+        "elasto_op_attention": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p],
+    }
+    for name, args in sig.items():
+        f = getattr(L, name)
+        f.argtypes = args
+        f.restype = c_int
+    L.elasto_last_error.argtypes = []
+    L.elasto_last_error.restype = ctypes.c_char_p
+    _lib = L
+    return L
+
+
+def elasto_last_error() -> str:
+    return (lib().elasto_last_error() or b"").decode()
+
+
+def _check(st: int, where: str) -> None:
+    if st != OK:
+        raise ElastoError(st, where, elasto_last_error())
+
+
+# ----------------------------------------------------------------------------
+# Marshalling helpers
+# ----------------------------------------------------------------------------
+
+class _Keep:
+    """Holds numpy arrays alive while their addresses are in a ctypes struct."""
+
+    def __init__(self):
+        self.items: List[object] = []
+
+    def arr(self, a, dtype) -> np.ndarray:
+        a = np.ascontiguousarray(a, dtype=dtype)
+        self.items.append(a)
+        return a
+
+    def i32(self, values) -> ctypes.POINTER(ctypes.c_int32):
+        a = self.arr(np.asarray(values, dtype=np.int32).reshape(-1), np.int32)
+        return a.ctypes.data_as(P_i32)
+
+
+def vit_desc(cfg, max_batch: int) -> ModelDesc:
+    return ModelDesc(ARCH_VIT, cfg.img, cfg.img, cfg.chans, cfg.patch, cfg.dim, cfg.heads, cfg.mlp, cfg.layers,
+                     cfg.classes, cfg.dtype, max_batch)
+
+
+def resnet_desc(cfg, max_batch: int) -> ModelDesc:
+    return ModelDesc(ARCH_RESNET50, cfg.img, cfg.img, cfg.chans, 0, 0, 0, 0, 0, cfg.classes, cfg.dtype, max_batch)
+
+
+def vit_mode_tables(keep: _Keep, tables: Sequence[Dict[str, Sequence[np.ndarray]]]):
+    arr = (ModeTables * len(tables))()
+    for m, t in enumerate(tables):
+        heads = [np.asarray(h, np.int32) for h in t["heads"]]
+        mlp = [np.asarray(f, np.int32) for f in t["mlp"]]
+        arr[m].heads_kept = keep.i32(np.concatenate(heads) if heads else [])
+        arr[m].n_heads_kept = keep.i32([len(h) for h in heads])
+        arr[m].mlp_kept = keep.i32(np.concatenate(mlp) if mlp else [])
+        arr[m].n_mlp_kept = keep.i32([len(f) for f in mlp])
+    return arr
+
+
+def resnet_mode_tables(keep: _Keep, tables):
+    arr = (ModeTables * len(tables))()
+    for m, t in enumerate(tables):
+        a = [np.asarray(x, np.int32) for x in t["a"]]
+        b = [np.asarray(x, np.int32) for x in t["b"]]
+        arr[m].conv_kept_a = keep.i32(np.concatenate(a))
+        arr[m].n_conv_a = keep.i32([len(x) for x in a])
+        arr[m].conv_kept_b = keep.i32(np.concatenate(b))
+        arr[m].n_conv_b = keep.i32([len(x) for x in b])
+    return arr
+
+
+def weights_struct(keep: _Keep, tensors: Sequence[np.ndarray]) -> Weights:
+    ptrs = (c_void_p * len(tensors))()
+    for i, t in enumerate(tensors):
+        a = np.ascontiguousarray(t)
+        keep.items.append(a)
+        ptrs[i] = a.ctypes.data
+    keep.items.append(ptrs)
+    return Weights(ptrs, len(tensors))
+
+
+# ----------------------------------------------------------------------------
+# C-ABI calls (same names)
+# ----------------------------------------------------------------------------
+
+def elasto_create(desc: ModelDesc, tensors: Sequence[np.ndarray], mode_tables, n_modes: int | None = None,
+                  keep: _Keep | None = None) -> int:
+    keep = keep or _Keep()
+    w = weights_struct(keep, tensors)
+    h = c_void_p()
+    n = len(mode_tables) if n_modes is None else n_modes
+    _check(lib().elasto_create(ctypes.byref(desc), ctypes.byref(w), mode_tables, n, ctypes.byref(h)),
+           "elasto_create")
+    return h.value
+
+
+def elasto_set_mode(h: int, mode: int) -> None:
+    _check(lib().elasto_set_mode(h, mode), "elasto_set_mode")
+
+
+def elasto_get_mode(h: int) -> int:
+    v = c_int()
+    _check(lib().elasto_get_mode(h, ctypes.byref(v)), "elasto_get_mode")
+    return v.value
+
+
+def elasto_forward(h: int, stream: int, images_ptr: int, batch: int, logits_ptr: int) -> None:
+    _check(lib().elasto_forward(h, stream, images_ptr, batch, logits_ptr), "elasto_forward")
+
+
+def elasto_forward_host(h: int, stream: int, images: np.ndarray, batch: int, logits: np.ndarray) -> None:
+    assert images.flags["C_CONTIGUOUS"] and logits.flags["C_CONTIGUOUS"] and logits.dtype == np.float32
+    _check(lib().elasto_forward_host(h, stream, images.ctypes.data, batch, logits.ctypes.data),
+           "elasto_forward_host")
+
+
+def elasto_sync_status(h: int, stream: int = 0) -> None:
+    _check(lib().elasto_sync_status(h, stream), "elasto_sync_status")
+
+
+def elasto_destroy(h: int) -> None:
+    _check(lib().elasto_destroy(h), "elasto_destroy")
+
+
+def elasto_query(h: int, what: int, mode: int = 0) -> int:
+    v = c_int64()
+    _check(lib().elasto_query(h, what, mode, ctypes.byref(v)), "elasto_query")
+    return v.value
+
+
+def elasto_debug_export_packed(h: int, mode: int, layer: int, which: int, out: np.ndarray) -> np.ndarray:
+    assert out.flags["C_CONTIGUOUS"]
+    _check(lib().elasto_debug_export_packed(h, mode, layer, which, out.ctypes.data, out.nbytes),
+           "elasto_debug_export_packed")
+    return out
+
+
+def elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status=0) -> None:
+    _check(lib().elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status), "elasto_op_gemm")
+
+
+def elasto_op_layernorm(stream, x, gamma, beta, y, rows, d) -> None:
+    _check(lib().elasto_op_layernorm(stream, x, gamma, beta, y, rows, d), "elasto_op_layernorm")
+
+
+def elasto_op_softmax(stream, x, y, rows, cols) -> None:
+    _check(lib().elasto_op_softmax(stream, x, y, rows, cols), "elasto_op_softmax")
+
+
+def elasto_op_attention(stream, qkv, out, batch, n, heads, status=0) -> None:
+    _check(lib().elasto_op_attention(stream, qkv, out, batch, n, heads, status), "elasto_op_attention")
+
+
+# ----------------------------------------------------------------------------
+# Owner object
+# ----------------------------------------------------------------------------
+
+class ElasticModel:
+    """One elastic model (libelasto handle) on the current CUDA device."""
+
+    def __init__(self, desc: ModelDesc, tensors: Sequence[np.ndarray], mode_tables, n_modes: int):
+        keep = _Keep()
+        self.desc = desc
+        self.n_modes = n_modes
+        self.handle = elasto_create(desc, tensors, mode_tables, n_modes, keep)
+
+    @classmethod
+    def vit(cls, cfg, weights: Dict[str, np.ndarray], tables, max_batch: int, names=None):
+        from . import synth
+        keep = _Keep()
+        names = names or synth.vit_weight_names(cfg)
+        mt = vit_mode_tables(keep, tables)
+        return cls(vit_desc(cfg, max_batch), [weights[k] for k in names], mt, len(tables))
+
+    @classmethod
+    def resnet(cls, cfg, weights: Dict[str, np.ndarray], tables, max_batch: int):
+        from . import synth
+        keep = _Keep()
+        mt = resnet_mode_tables(keep, tables)
+        return cls(resnet_desc(cfg, max_batch), [weights[k] for k in synth.resnet_weight_names(cfg)], mt,
+                   len(tables))
+
+    def set_mode(self, mode: int) -> None:
+        elasto_set_mode(self.handle, mode)
+
+    @property
+    def mode(self) -> int:
+        return elasto_get_mode(self.handle)
+
+    def forward(self, stream: int, images_ptr: int, batch: int, logits_ptr: int) -> None:
+        elasto_forward(self.handle, stream, images_ptr, batch, logits_ptr)
+
+    def forward_host(self, images: np.ndarray, logits: np.ndarray, stream: int = 0) -> None:
+        elasto_forward_host(self.handle, stream, images, images.shape[0], logits)
+
+    def sync_status(self, stream: int = 0) -> None:
+        elasto_sync_status(self.handle, stream)
+
+    def query(self, what: int, mode: int = 0) -> int:
+        return elasto_query(self.handle, what, mode)
+
+    def export_packed(self, mode: int, layer: int, which: int, out: np.ndarray) -> np.ndarray:
+        return elasto_debug_export_packed(self.handle, mode, layer, which, out)
+
+    def close(self) -> None:
+        if self.handle:
+            elasto_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()

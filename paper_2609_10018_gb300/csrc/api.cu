@@ -1,0 +1,722 @@
+// C-ABI of libelasto: elastic model handle, create-time packing of every
+// descendant network (DN), O(1) mode switching, and the forward pass.
+//
+// Section 4.3: all DNs share one parameter set and differ in which heads /
+// MLP channels / conv channels they keep. The structured masks of Eq. 4, 6
+// and 7 zero whole rows or columns; computing with zeros is wasted work, so at
+// create time each mode's kept rows/columns are gathered into contiguous
+// packed matrices (the kept-index tables play the role of the paper's
+// "pruning metadata", Section 4.1-4.2). A mode switch then only swaps which
+// packed set the next forward reads (Section 6.2 measures the paper's own
+// switch cost): no weight moves on the request path.
+#include <stdio.h>
+
+#include <algorithm>
+#include <atomic>
+#include <memory>
+#include <mutex>
+#include <vector>
+
+#include "common.h"
+#include "elasto_internal.h"
+
+namespace elasto {
+
+const char* last_error_cstr();
+
+namespace {
+
+constexpr size_t kAlign = 1024;
+
+struct Bump {
+  size_t off = 0;
+  size_t take(size_t bytes) {
+    off = (off + kAlign - 1) / kAlign * kAlign;
+    const size_t r = off;
+    off += bytes;
+    return r;
+  }
+};
+
+size_t dtype_size(int dt) { return dt == ELASTO_BF16 ? 2 : 4; }
+
+bool tables_ok(const int32_t* idx, int n, int limit) {
+  for (int i = 0; i < n; ++i) {
+    if (idx[i] < 0 || idx[i] >= limit) return false;
+    if (i > 0 && idx[i] <= idx[i - 1]) return false;
+  }
+  return true;
+}
+
+std::once_flag g_attr_once[64];
+cudaError_t g_attr_err[64];
+
+}  // namespace
+
+cudaError_t ensure_kernel_attributes() {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::call_once(g_attr_once[dev], [dev] {
+    cudaError_t r = gemm_init_attributes();
+    if (r == cudaSuccess) r = attn_init_attributes();
+    g_attr_err[dev] = r;
+  });
+  return g_attr_err[dev];
+}
+
+elasto_status check_device() {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+  if (major != 10 || minor != 3) {
+    char buf[128];
+    snprintf(buf, sizeof buf, "libelasto is built for sm_103a (GB300); device %d is sm_%d%d", dev, major, minor);
+    set_error(buf);
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  e = ensure_kernel_attributes();
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute");
+  return ELASTO_OK;
+}
+
+}  // namespace elasto
+
+using namespace elasto;
+
+// ============================================================================
+// ViT
+// ============================================================================
+namespace {
+
+struct VitLayerPack {
+  int w = 0;       // kept heads * 64
+  int f = 0;       // kept MLP channels
+  int f_pad = 0;   // f rounded up to a multiple of 8 (zero rows/cols; GELU(0) = 0)
+  bf16* qkv_w = nullptr;
+  float* qkv_b = nullptr;
+  bf16* proj_w = nullptr;
+  bf16* fc1_w = nullptr;
+  float* fc1_b = nullptr;
+  bf16* fc2_w = nullptr;
+  GemmPlan qkv, proj, fc1, fc2;
+  AttnPlan attn;
+};
+
+struct VitMode {
+  std::vector<VitLayerPack> layers;
+  size_t packed_bytes = 0;
+  int64_t macs = 0;
+  int launches = 0;
+};
+
+}  // namespace
+
+struct elasto_s {
+  elasto_model_desc d{};
+  int dev = 0;
+  int n = 0, np = 0, kpe = 0;
+  char* arena = nullptr;
+  size_t arena_bytes = 0, shared_bytes = 0, workspace_bytes = 0;
+  // shared (mode-independent) parameters
+  bf16* patch_w = nullptr;
+  float *patch_b = nullptr, *cls = nullptr, *pos = nullptr, *norm_w = nullptr, *norm_b = nullptr;
+  float *head_w = nullptr, *head_b = nullptr;
+  std::vector<float*> ln1_w, ln1_b, proj_b, ln2_w, ln2_b, fc2_b;
+  // workspace
+  float* X = nullptr;
+  bf16 *Y = nullptr, *QKV = nullptr, *O = nullptr, *H = nullptr, *P = nullptr;
+  void* img_stage = nullptr;
+  float* logit_stage = nullptr;
+  int* status = nullptr;
+  GemmPlan patch;
+  std::vector<VitMode> modes;
+  std::atomic<int> cur{0};
+  // CNN state lives behind this pointer (null for ViT)
+  CnnModel* cnn = nullptr;
+};
+
+namespace {
+
+elasto_status vit_validate(const elasto_model_desc* d) {
+  if (d->img_h <= 0 || d->img_h != d->img_w || d->img_c <= 0 || d->patch <= 0 || d->img_h % d->patch != 0 ||
+      d->dim <= 0 || d->heads <= 0 || d->dim != d->heads * 64 || d->mlp <= 0 || d->layers <= 0 ||
+      d->classes <= 0) {
+    set_error("elasto_create: inconsistent ViT descriptor (need img_h == img_w, patch | img_h, dim == 64 * heads)");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int np = (d->img_h / d->patch) * (d->img_w / d->patch);
+  const int kpe = d->patch * d->patch * d->img_c;
+  if (np + 1 > 256) {
+    set_error("elasto_create: at most 256 tokens (255 patches) are supported");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  if (kpe % 8 != 0 || d->dim % 64 != 0 || d->dim > 1024) {
+    set_error("elasto_create: need patch*patch*channels % 8 == 0 and dim a multiple of 64 up to 1024");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  return ELASTO_OK;
+}
+
+elasto_status vit_validate_tables(const elasto_model_desc* d, const elasto_mode_tables* modes, int n_modes) {
+  for (int m = 0; m < n_modes; ++m) {
+    const elasto_mode_tables& t = modes[m];
+    if (!t.n_heads_kept || !t.n_mlp_kept) {
+      set_error("elasto_create: mode " + std::to_string(m) + " has no count arrays");
+      return ELASTO_ERR_INVALID_ARG;
+    }
+    size_t ho = 0, fo = 0;
+    for (int l = 0; l < d->layers; ++l) {
+      const int nh = t.n_heads_kept[l], nf = t.n_mlp_kept[l];
+      if (nh < 0 || nh > d->heads || nf < 0 || nf > d->mlp) {
+        set_error("elasto_create: mode " + std::to_string(m) + " layer " + std::to_string(l) +
+                  ": kept count out of range");
+        return ELASTO_ERR_BAD_TABLE;
+      }
+      if ((nh > 0 && !t.heads_kept) || (nf > 0 && !t.mlp_kept)) {
+        set_error("elasto_create: mode " + std::to_string(m) + ": null index table");
+        return ELASTO_ERR_INVALID_ARG;
+      }
+      if ((nh > 0 && !tables_ok(t.heads_kept + ho, nh, d->heads)) ||
+          (nf > 0 && !tables_ok(t.mlp_kept + fo, nf, d->mlp))) {
+        set_error("elasto_create: mode " + std::to_string(m) + " layer " + std::to_string(l) +
+                  ": kept indices must be strictly increasing and in range");
+        return ELASTO_ERR_BAD_TABLE;
+      }
+      ho += nh;
+      fo += nf;
+    }
+  }
+  return ELASTO_OK;
+}
+
+// Free-on-exit temporary device buffer.
+struct DevTemp {
+  void* p = nullptr;
+  ~DevTemp() {
+    if (p) cudaFree(p);
+  }
+};
+
+// Everything that can be checked on the host, before any CUDA call.
+elasto_status vit_check_inputs(const elasto_model_desc* d, const elasto_weights* wts,
+                               const elasto_mode_tables* modes, int n_modes) {
+  elasto_status st = vit_validate(d);
+  if (st != ELASTO_OK) return st;
+  if (wts->n_tensors != 8 + 12 * d->layers) {
+    set_error("elasto_create: ViT expects 8 + 12 * layers weight tensors, got " + std::to_string(wts->n_tensors));
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  for (int i = 0; i < wts->n_tensors; ++i)
+    if (!wts->tensors[i]) {
+      set_error("elasto_create: weight tensor " + std::to_string(i) + " is null");
+      return ELASTO_ERR_INVALID_ARG;
+    }
+  return vit_validate_tables(d, modes, n_modes);
+}
+
+elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, const elasto_mode_tables* modes,
+                         int n_modes, elasto_s* h) {
+  elasto_status st = vit_check_inputs(d, wts, modes, n_modes);
+  if (st != ELASTO_OK) return st;
+  const int L = d->layers, D = d->dim, F = d->mlp, C = d->classes, Bm = d->max_batch;
+  const int P = d->patch, np = (d->img_h / P) * (d->img_w / P), n = np + 1, kpe = P * P * d->img_c;
+  h->n = n;
+  h->np = np;
+  h->kpe = kpe;
+
+  // ---------------------------------------------------------------- layout
+  Bump bump;
+  const size_t o_patch_w = bump.take(size_t(D) * kpe * 2);
+  const size_t o_patch_b = bump.take(D * 4), o_cls = bump.take(D * 4), o_pos = bump.take(size_t(n) * D * 4);
+  std::vector<size_t> o_l(6 * L);
+  for (int l = 0; l < L; ++l)
+    for (int k = 0; k < 6; ++k) o_l[6 * l + k] = bump.take(D * 4);
+  const size_t o_norm_w = bump.take(D * 4), o_norm_b = bump.take(D * 4);
+  const size_t o_head_w = bump.take(size_t(C) * D * 4), o_head_b = bump.take(C * 4);
+  h->shared_bytes = bump.off;
+
+  h->modes.assign(n_modes, VitMode{});
+  struct Off {
+    size_t qkv_w, qkv_b, proj_w, fc1_w, fc1_b, fc2_w;
+  };
+  std::vector<std::vector<Off>> offs(n_modes, std::vector<Off>(L));
+  int wmax = 0, fmax = 0;
+  for (int m = 0; m < n_modes; ++m) {
+    const size_t start = bump.off;
+    h->modes[m].layers.resize(L);
+    for (int l = 0; l < L; ++l) {
+      VitLayerPack& lp = h->modes[m].layers[l];
+      lp.w = 64 * modes[m].n_heads_kept[l];
+      lp.f = modes[m].n_mlp_kept[l];
+      lp.f_pad = (lp.f + 7) / 8 * 8;
+      wmax = std::max(wmax, lp.w);
+      fmax = std::max(fmax, lp.f_pad);
+      Off& o = offs[m][l];
+      o.qkv_w = bump.take(size_t(3) * lp.w * D * 2);
+      o.qkv_b = bump.take(size_t(3) * lp.w * 4);
+      o.proj_w = bump.take(size_t(D) * lp.w * 2);
+      o.fc1_w = bump.take(size_t(lp.f_pad) * D * 2);
+      o.fc1_b = bump.take(size_t(lp.f_pad) * 4);
+      o.fc2_w = bump.take(size_t(D) * lp.f_pad * 2);
+    }
+    h->modes[m].packed_bytes = bump.off - start;
+  }
+  const size_t ws_start = bump.off;
+  const size_t rows = size_t(Bm) * n;
+  const size_t o_X = bump.take(rows * D * 4), o_Y = bump.take(rows * D * 2);
+  const size_t o_QKV = bump.take(rows * 3 * std::max(wmax, 64) * 2), o_O = bump.take(rows * std::max(wmax, 64) * 2);
+  const size_t o_H = bump.take(rows * std::max(fmax, 8) * 2), o_P = bump.take(size_t(Bm) * np * kpe * 2);
+  const size_t img_bytes = size_t(Bm) * d->img_h * d->img_w * d->img_c * dtype_size(d->weight_dtype);
+  const size_t o_img = bump.take(img_bytes), o_logit = bump.take(size_t(Bm) * C * 4);
+  const size_t o_status = bump.take(64);
+  h->workspace_bytes = bump.off - ws_start;
+  h->arena_bytes = bump.off;
+
+  cudaError_t e = cudaMalloc(&h->arena, h->arena_bytes);
+  if (e != cudaSuccess) {
+    h->arena = nullptr;
+    cudaGetLastError();
+    set_error("elasto_create: cudaMalloc of " + std::to_string(h->arena_bytes) + " bytes failed");
+    return ELASTO_ERR_OOM;
+  }
+  char* A = h->arena;
+  h->patch_w = reinterpret_cast<bf16*>(A + o_patch_w);
+  h->patch_b = reinterpret_cast<float*>(A + o_patch_b);
+  h->cls = reinterpret_cast<float*>(A + o_cls);
+  h->pos = reinterpret_cast<float*>(A + o_pos);
+  for (int l = 0; l < L; ++l) {
+    h->ln1_w.push_back(reinterpret_cast<float*>(A + o_l[6 * l + 0]));
+    h->ln1_b.push_back(reinterpret_cast<float*>(A + o_l[6 * l + 1]));
+    h->proj_b.push_back(reinterpret_cast<float*>(A + o_l[6 * l + 2]));
+    h->ln2_w.push_back(reinterpret_cast<float*>(A + o_l[6 * l + 3]));
+    h->ln2_b.push_back(reinterpret_cast<float*>(A + o_l[6 * l + 4]));
+    h->fc2_b.push_back(reinterpret_cast<float*>(A + o_l[6 * l + 5]));
+  }
+  h->norm_w = reinterpret_cast<float*>(A + o_norm_w);
+  h->norm_b = reinterpret_cast<float*>(A + o_norm_b);
+  h->head_w = reinterpret_cast<float*>(A + o_head_w);
+  h->head_b = reinterpret_cast<float*>(A + o_head_b);
+  h->X = reinterpret_cast<float*>(A + o_X);
+  h->Y = reinterpret_cast<bf16*>(A + o_Y);
+  h->QKV = reinterpret_cast<bf16*>(A + o_QKV);
+  h->O = reinterpret_cast<bf16*>(A + o_O);
+  h->H = reinterpret_cast<bf16*>(A + o_H);
+  h->P = reinterpret_cast<bf16*>(A + o_P);
+  h->img_stage = A + o_img;
+  h->logit_stage = reinterpret_cast<float*>(A + o_logit);
+  h->status = reinterpret_cast<int*>(A + o_status);
+  for (int m = 0; m < n_modes; ++m)
+    for (int l = 0; l < L; ++l) {
+      VitLayerPack& lp = h->modes[m].layers[l];
+      const Off& o = offs[m][l];
+      lp.qkv_w = reinterpret_cast<bf16*>(A + o.qkv_w);
+      lp.qkv_b = reinterpret_cast<float*>(A + o.qkv_b);
+      lp.proj_w = reinterpret_cast<bf16*>(A + o.proj_w);
+      lp.fc1_w = reinterpret_cast<bf16*>(A + o.fc1_w);
+      lp.fc1_b = reinterpret_cast<float*>(A + o.fc1_b);
+      lp.fc2_w = reinterpret_cast<bf16*>(A + o.fc2_w);
+    }
+  ELASTO_CUDA_TRY(cudaMemset(h->arena, 0, h->arena_bytes));
+
+  // ---------------------------------------------------------------- upload
+  const int dt = d->weight_dtype;
+  const size_t es = dtype_size(dt);
+  auto W = [&](int i) { return wts->tensors[i]; };
+  // temp: raw upload buffer + canonical bf16 + canonical fp32 bias + index list
+  const size_t max_mat = std::max({size_t(3) * D * D, size_t(F) * D, size_t(D) * kpe});
+  DevTemp raw, canon, canon_b, idxbuf;
+  ELASTO_CUDA_TRY(cudaMalloc(&raw.p, max_mat * 4 + size_t(n) * D * 4 + size_t(C) * D * 4));
+  ELASTO_CUDA_TRY(cudaMalloc(&canon.p, max_mat * 2));
+  ELASTO_CUDA_TRY(cudaMalloc(&canon_b.p, size_t(std::max(3 * D, F)) * 4));
+  ELASTO_CUDA_TRY(cudaMalloc(&idxbuf.p, size_t(std::max(3 * D, F) + 64) * 4));
+  cudaStream_t s = 0;
+
+  auto up_f32 = [&](const void* src, size_t count, float* dst) -> elasto_status {
+    ELASTO_CUDA_TRY(cudaMemcpy(raw.p, src, count * es, cudaMemcpyHostToDevice));
+    ELASTO_CUDA_TRY(convert_to_f32(raw.p, dt, count, dst, s));
+    return ELASTO_OK;
+  };
+  auto up_bf16 = [&](const void* src, size_t count, bf16* dst) -> elasto_status {
+    ELASTO_CUDA_TRY(cudaMemcpy(raw.p, src, count * es, cudaMemcpyHostToDevice));
+    ELASTO_CUDA_TRY(convert_to_bf16(raw.p, dt, count, dst, s));
+    return ELASTO_OK;
+  };
+#define UP(expr)                       \
+  do {                                 \
+    elasto_status s_ = (expr);         \
+    if (s_ != ELASTO_OK) return s_;    \
+  } while (0)
+
+  // patch_w [d, C, P, P] -> packed [d, (ky, kx, c)] to match NHWC patch rows
+  {
+    std::vector<char> re(size_t(D) * kpe * es);
+    const char* src = static_cast<const char*>(W(0));
+    const int Cc = d->img_c;
+    for (int o = 0; o < D; ++o)
+      for (int c = 0; c < Cc; ++c)
+        for (int ky = 0; ky < P; ++ky)
+          for (int kx = 0; kx < P; ++kx) {
+            const size_t si = ((size_t(o) * Cc + c) * P + ky) * P + kx;
+            const size_t di = size_t(o) * kpe + (size_t(ky) * P + kx) * Cc + c;
+            memcpy(re.data() + di * es, src + si * es, es);
+          }
+    UP(up_bf16(re.data(), size_t(D) * kpe, h->patch_w));
+  }
+  UP(up_f32(W(1), D, h->patch_b));
+  UP(up_f32(W(2), D, h->cls));
+  UP(up_f32(W(3), size_t(n) * D, h->pos));
+  const int base_final = 4 + 12 * L;
+  UP(up_f32(W(base_final + 0), D, h->norm_w));
+  UP(up_f32(W(base_final + 1), D, h->norm_b));
+  UP(up_f32(W(base_final + 2), size_t(C) * D, h->head_w));
+  UP(up_f32(W(base_final + 3), C, h->head_b));
+
+  std::vector<int32_t> idx;
+  for (int l = 0; l < L; ++l) {
+    const int t0 = 4 + 12 * l;  // ln1_w, ln1_b, qkv_w, qkv_b, proj_w, proj_b, ln2_w, ln2_b, fc1_w, fc1_b, fc2_w, fc2_b
+    UP(up_f32(W(t0 + 0), D, h->ln1_w[l]));
+    UP(up_f32(W(t0 + 1), D, h->ln1_b[l]));
+    UP(up_f32(W(t0 + 5), D, h->proj_b[l]));
+    UP(up_f32(W(t0 + 6), D, h->ln2_w[l]));
+    UP(up_f32(W(t0 + 7), D, h->ln2_b[l]));
+    UP(up_f32(W(t0 + 11), D, h->fc2_b[l]));
+    bf16* cw = static_cast<bf16*>(canon.p);
+    float* cb = static_cast<float*>(canon_b.p);
+    int32_t* di = static_cast<int32_t*>(idxbuf.p);
+    // qkv: rows {blk * d + j * 64 + r}
+    UP(up_bf16(W(t0 + 2), size_t(3) * D * D, cw));
+    UP(up_f32(W(t0 + 3), size_t(3) * D, cb));
+    for (int m = 0; m < n_modes; ++m) {
+      VitLayerPack& lp = h->modes[m].layers[l];
+      if (lp.w == 0) continue;
+      size_t ho = 0;
+      for (int k = 0; k < l; ++k) ho += modes[m].n_heads_kept[k];
+      const int32_t* hk = modes[m].heads_kept + ho;
+      idx.clear();
+      for (int blk = 0; blk < 3; ++blk)
+        for (int j = 0; j < lp.w / 64; ++j)
+          for (int r = 0; r < 64; ++r) idx.push_back(blk * D + hk[j] * 64 + r);
+      ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, int(idx.size()), lp.qkv_w, s));
+      ELASTO_CUDA_TRY(gather_f32(cb, di, int(idx.size()), lp.qkv_b, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    // proj: columns {j * 64 + r}
+    UP(up_bf16(W(t0 + 4), size_t(D) * D, cw));
+    for (int m = 0; m < n_modes; ++m) {
+      VitLayerPack& lp = h->modes[m].layers[l];
+      if (lp.w == 0) continue;
+      size_t ho = 0;
+      for (int k = 0; k < l; ++k) ho += modes[m].n_heads_kept[k];
+      const int32_t* hk = modes[m].heads_kept + ho;
+      idx.clear();
+      for (int j = 0; j < lp.w / 64; ++j)
+        for (int r = 0; r < 64; ++r) idx.push_back(hk[j] * 64 + r);
+      ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, D, di, int(idx.size()), lp.proj_w, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    // fc1: rows F (padding rows stay zero), b1 entries F
+    UP(up_bf16(W(t0 + 8), size_t(F) * D, cw));
+    UP(up_f32(W(t0 + 9), F, cb));
+    for (int m = 0; m < n_modes; ++m) {
+      VitLayerPack& lp = h->modes[m].layers[l];
+      if (lp.f == 0) continue;
+      size_t fo = 0;
+      for (int k = 0; k < l; ++k) fo += modes[m].n_mlp_kept[k];
+      ELASTO_CUDA_TRY(cudaMemcpy(di, modes[m].mlp_kept + fo, size_t(lp.f) * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, lp.f, lp.fc1_w, s));
+      ELASTO_CUDA_TRY(gather_f32(cb, di, lp.f, lp.fc1_b, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    // fc2: columns F into [d, f_pad] (padding columns zero)
+    UP(up_bf16(W(t0 + 10), size_t(D) * F, cw));
+    for (int m = 0; m < n_modes; ++m) {
+      VitLayerPack& lp = h->modes[m].layers[l];
+      if (lp.f == 0) continue;
+      size_t fo = 0;
+      for (int k = 0; k < l; ++k) fo += modes[m].n_mlp_kept[k];
+      idx.assign(modes[m].mlp_kept + fo, modes[m].mlp_kept + fo + lp.f);
+      for (int k = lp.f; k < lp.f_pad; ++k) idx.push_back(-1);
+      ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, F, di, lp.f_pad, lp.fc2_w, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+  }
+#undef UP
+  ELASTO_CUDA_TRY(cudaDeviceSynchronize());
+
+  // ---------------------------------------------------------------- plans
+  const int Mcap = Bm * n;
+  st = gemm_plan(&h->patch, h->P, Bm * np, h->patch_w, D, kpe, h->patch_b, h->X, D, EPI_PATCH_POS_F32, h->status);
+  if (st != ELASTO_OK) return st;
+  h->patch.args.patches = np;
+  h->patch.args.tokens = n;
+  h->patch.args.pos = h->pos;
+  const int64_t lin_patch = int64_t(np) * D * kpe + int64_t(D) * C;
+  for (int m = 0; m < n_modes; ++m) {
+    VitMode& vm = h->modes[m];
+    vm.macs = lin_patch;
+    vm.launches = 3;  // patchify, patch GEMM, head
+    for (int l = 0; l < L; ++l) {
+      VitLayerPack& lp = vm.layers[l];
+      vm.macs += int64_t(n) * D * 3 * lp.w + 2 * int64_t(n) * n * lp.w + int64_t(n) * lp.w * D +
+                 2 * int64_t(n) * D * lp.f;
+      vm.launches += 2;  // two LayerNorms
+      if (lp.w > 0) {
+        st = gemm_plan(&lp.qkv, h->Y, Mcap, lp.qkv_w, 3 * lp.w, D, lp.qkv_b, h->QKV, 3 * lp.w, EPI_BIAS_BF16,
+                       h->status);
+        if (st != ELASTO_OK) return st;
+        st = attn_plan(&lp.attn, h->QKV, h->O, Bm, n, lp.w / 64, h->status);
+        if (st != ELASTO_OK) return st;
+        vm.launches += 2;
+      }
+      st = gemm_plan(&lp.proj, h->O, Mcap, lp.proj_w, D, lp.w, h->proj_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status);
+      if (st != ELASTO_OK) return st;
+      if (lp.f > 0) {
+        st = gemm_plan(&lp.fc1, h->Y, Mcap, lp.fc1_w, lp.f_pad, D, lp.fc1_b, h->H, lp.f_pad, EPI_BIAS_GELU_BF16,
+                       h->status);
+        if (st != ELASTO_OK) return st;
+        vm.launches += 1;
+      }
+      st = gemm_plan(&lp.fc2, h->H, Mcap, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status);
+      if (st != ELASTO_OK) return st;
+      vm.launches += 2;
+    }
+  }
+  return ELASTO_OK;
+}
+
+elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int batch, float* logits) {
+  const elasto_model_desc& d = h->d;
+  const VitMode& vm = h->modes[h->cur.load(std::memory_order_acquire)];
+  const int n = h->n, D = d.dim, M = batch * n;
+  ELASTO_CUDA_TRY(
+      patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, h->X, h->cls, h->pos, D, s));
+  ELASTO_CUDA_TRY(gemm_launch(h->patch, batch * h->np, s));
+  for (int l = 0; l < d.layers; ++l) {
+    const VitLayerPack& lp = vm.layers[l];
+    ELASTO_CUDA_TRY(layernorm_launch(h->X, h->ln1_w[l], h->ln1_b[l], h->Y, M, D, s));
+    if (lp.w > 0) {
+      ELASTO_CUDA_TRY(gemm_launch(lp.qkv, M, s));
+      ELASTO_CUDA_TRY(attn_launch(lp.attn, batch, s));
+    }
+    ELASTO_CUDA_TRY(gemm_launch(lp.proj, M, s));
+    ELASTO_CUDA_TRY(layernorm_launch(h->X, h->ln2_w[l], h->ln2_b[l], h->Y, M, D, s));
+    if (lp.f > 0) ELASTO_CUDA_TRY(gemm_launch(lp.fc1, M, s));
+    ELASTO_CUDA_TRY(gemm_launch(lp.fc2, M, s));
+  }
+  ELASTO_CUDA_TRY(head_launch(h->X, batch, n, D, h->norm_w, h->norm_b, h->head_w, h->head_b, d.classes, logits, s));
+  return ELASTO_OK;
+}
+
+}  // namespace
+
+// ============================================================================
+// Exported C-ABI
+// ============================================================================
+extern "C" {
+
+elasto_status elasto_create(const elasto_model_desc* desc, const elasto_weights* weights,
+                            const elasto_mode_tables* modes, int n_modes, elasto_t* out) {
+  clear_error();
+  if (!desc || !weights || !weights->tensors || !modes || n_modes <= 0 || !out) {
+    set_error("elasto_create: null argument or n_modes <= 0");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  *out = nullptr;
+  if (desc->max_batch <= 0 || (desc->weight_dtype != ELASTO_F32 && desc->weight_dtype != ELASTO_BF16)) {
+    set_error("elasto_create: max_batch must be >= 1 and weight_dtype ELASTO_F32 or ELASTO_BF16");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (desc->arch != ELASTO_ARCH_VIT && desc->arch != ELASTO_ARCH_RESNET50) {
+    set_error("elasto_create: unknown arch");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  elasto_status st = desc->arch == ELASTO_ARCH_VIT ? vit_check_inputs(desc, weights, modes, n_modes)
+                                                   : cnn_check_inputs(desc, weights, modes, n_modes);
+  if (st != ELASTO_OK) return st;
+  st = check_device();
+  if (st != ELASTO_OK) return st;
+  std::unique_ptr<elasto_s> h(new elasto_s());
+  h->d = *desc;
+  cudaGetDevice(&h->dev);
+  if (desc->arch == ELASTO_ARCH_VIT) {
+    st = vit_create(desc, weights, modes, n_modes, h.get());
+  } else {
+    h->cnn = cnn_new();
+    st = cnn_create(desc, weights, modes, n_modes, h->cnn);
+  }
+  if (st != ELASTO_OK) {
+    cudaDeviceSynchronize();
+    if (h->arena) cudaFree(h->arena);
+    if (h->cnn) cnn_destroy(h->cnn);
+    return st;
+  }
+  h->cur.store(0);
+  *out = h.release();
+  return ELASTO_OK;
+}
+
+elasto_status elasto_set_mode(elasto_t h, int mode) {
+  if (!h) {
+    set_error("elasto_set_mode: null handle");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int nm = h->cnn ? cnn_n_modes(h->cnn) : static_cast<int>(h->modes.size());
+  if (mode < 0 || mode >= nm) {
+    set_error("elasto_set_mode: mode " + std::to_string(mode) + " out of range [0, " + std::to_string(nm) + ")");
+    return ELASTO_ERR_BAD_MODE;
+  }
+  h->cur.store(mode, std::memory_order_release);
+  return ELASTO_OK;
+}
+
+elasto_status elasto_get_mode(elasto_t h, int* mode) {
+  if (!h || !mode) {
+    set_error("elasto_get_mode: null argument");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  *mode = h->cur.load(std::memory_order_acquire);
+  return ELASTO_OK;
+}
+
+elasto_status elasto_forward(elasto_t h, void* stream, const void* images, int batch, float* logits) {
+  if (!h || !images || !logits) {
+    set_error("elasto_forward: null argument");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (batch < 1 || batch > h->d.max_batch) {
+    set_error("elasto_forward: batch " + std::to_string(batch) + " outside [1, max_batch]");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (h->cnn) return cnn_forward(h->cnn, h->cur.load(std::memory_order_acquire), s, images, batch, logits);
+  return vit_forward(h, s, images, batch, logits);
+}
+
+elasto_status elasto_forward_host(elasto_t h, void* stream, const void* images_host, int batch,
+                                  float* logits_host) {
+  if (!h || !images_host || !logits_host) {
+    set_error("elasto_forward_host: null argument");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (batch < 1 || batch > h->d.max_batch) {
+    set_error("elasto_forward_host: batch outside [1, max_batch]");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  void* img_dev = h->cnn ? cnn_image_stage(h->cnn) : h->img_stage;
+  float* logit_dev = h->cnn ? cnn_logit_stage(h->cnn) : h->logit_stage;
+  const size_t ib = size_t(batch) * h->d.img_h * h->d.img_w * h->d.img_c * dtype_size(h->d.weight_dtype);
+  ELASTO_CUDA_TRY(cudaMemcpyAsync(img_dev, images_host, ib, cudaMemcpyHostToDevice, s));
+  elasto_status st = elasto_forward(h, stream, img_dev, batch, logit_dev);
+  if (st != ELASTO_OK) return st;
+  ELASTO_CUDA_TRY(cudaMemcpyAsync(logits_host, logit_dev, size_t(batch) * h->d.classes * 4, cudaMemcpyDeviceToHost, s));
+  ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+  return ELASTO_OK;
+}
+
+elasto_status elasto_sync_status(elasto_t h, void* stream) {
+  if (!h) {
+    set_error("elasto_sync_status: null handle");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  ELASTO_CUDA_TRY(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)));
+  int* sw = h->cnn ? cnn_status_word(h->cnn) : h->status;
+  int v = 0;
+  ELASTO_CUDA_TRY(cudaMemcpy(&v, sw, sizeof v, cudaMemcpyDeviceToHost));
+  if (v != 0) {
+    ELASTO_CUDA_TRY(cudaMemset(sw, 0, sizeof v));
+    set_error("device status word: a bounded device-side wait gave up");
+    return static_cast<elasto_status>(v);
+  }
+  return ELASTO_OK;
+}
+
+elasto_status elasto_destroy(elasto_t h) {
+  if (!h) {
+    set_error("elasto_destroy: null handle");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  cudaDeviceSynchronize();
+  if (h->arena) cudaFree(h->arena);
+  if (h->cnn) cnn_destroy(h->cnn);
+  delete h;
+  return ELASTO_OK;
+}
+
+const char* elasto_last_error(void) { return last_error_cstr(); }
+
+elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value) {
+  if (!h || !value) {
+    set_error("elasto_query: null argument");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (h->cnn) return cnn_query(h->cnn, what, mode, value);
+  const int nm = static_cast<int>(h->modes.size());
+  const bool needs_mode = what == ELASTO_Q_PACKED_BYTES || what == ELASTO_Q_MODE_MACS || what == ELASTO_Q_LAUNCHES;
+  if (needs_mode && (mode < 0 || mode >= nm)) {
+    set_error("elasto_query: bad mode");
+    return ELASTO_ERR_BAD_MODE;
+  }
+  switch (what) {
+    case ELASTO_Q_N_MODES: *value = nm; break;
+    case ELASTO_Q_PACKED_BYTES: *value = int64_t(h->modes[mode].packed_bytes); break;
+    case ELASTO_Q_SHARED_BYTES: *value = int64_t(h->shared_bytes); break;
+    case ELASTO_Q_WORKSPACE_BYTES: *value = int64_t(h->workspace_bytes); break;
+    case ELASTO_Q_ARENA_BYTES: *value = int64_t(h->arena_bytes); break;
+    case ELASTO_Q_MODE_MACS: *value = h->modes[mode].macs; break;
+    case ELASTO_Q_LAUNCHES: *value = h->modes[mode].launches; break;
+    default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
+  }
+  return ELASTO_OK;
+}
+
+elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int which, void* host_dst, size_t bytes) {
+  if (!h || !host_dst) {
+    set_error("elasto_debug_export_packed: null argument");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (h->cnn) return cnn_export_packed(h->cnn, mode, layer, which, host_dst, bytes);
+  if (mode < 0 || mode >= static_cast<int>(h->modes.size())) {
+    set_error("elasto_debug_export_packed: bad mode");
+    return ELASTO_ERR_BAD_MODE;
+  }
+  if (layer < 0 || layer >= h->d.layers || which < 0 || which > 5) {
+    set_error("elasto_debug_export_packed: bad layer or buffer index");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const VitLayerPack& lp = h->modes[mode].layers[layer];
+  const size_t D = h->d.dim;
+  size_t need = 0;
+  const void* src = nullptr;
+  switch (which) {
+    case 0: need = size_t(3) * lp.w * D * 2; src = lp.qkv_w; break;
+    case 1: need = size_t(3) * lp.w * 4; src = lp.qkv_b; break;
+    case 2: need = D * lp.w * 2; src = lp.proj_w; break;
+    case 3: need = size_t(lp.f) * D * 2; src = lp.fc1_w; break;
+    case 4: need = size_t(lp.f) * 4; src = lp.fc1_b; break;
+    case 5: need = D * lp.f * 2; src = lp.fc2_w; break;
+  }
+  if (bytes != need) {
+    set_error("elasto_debug_export_packed: expected " + std::to_string(need) + " bytes");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (need == 0) return ELASTO_OK;
+  if (which == 5) {
+    // stored [d, f_pad]; export [d, f]
+    ELASTO_CUDA_TRY(cudaMemcpy2D(host_dst, size_t(lp.f) * 2, src, size_t(lp.f_pad) * 2, size_t(lp.f) * 2, D,
+                                 cudaMemcpyDeviceToHost));
+  } else {
+    ELASTO_CUDA_TRY(cudaMemcpy(host_dst, src, need, cudaMemcpyDeviceToHost));
+  }
+  return ELASTO_OK;
+}
+
+}  // extern "C"

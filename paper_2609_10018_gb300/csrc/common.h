@@ -1,0 +1,114 @@
+// Internal declarations shared by the translation units of libelasto.
+#pragma once
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+
+#include "elasto.h"
+#include "elasto_ops.h"
+
+namespace elasto {
+
+using bf16 = __nv_bfloat16;
+
+// ---------------------------------------------------------------- errors
+void set_error(const std::string& msg);
+void clear_error();
+elasto_status cuda_fail(cudaError_t e, const char* what);  // records "<what>: <cuda msg>"
+
+#define ELASTO_CUDA_TRY(expr)                                  \
+  do {                                                         \
+    cudaError_t e_ = (expr);                                   \
+    if (e_ != cudaSuccess) return ::elasto::cuda_fail(e_, #expr); \
+  } while (0)
+
+// ---------------------------------------------------------------- device facts
+int num_sms();  // of the current device
+
+// ---------------------------------------------------------------- TMA maps
+// 2-D bf16 tensor [outer][inner] (inner contiguous, row stride in bytes),
+// box {box_inner, box_outer}, 128-byte swizzle, out-of-bounds reads as zero.
+bool encode_tmap_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_stride_bytes,
+                    uint32_t box_inner, uint32_t box_outer);
+// 3-D bf16 tensor [d2][d1][d0] with byte strides s1 (between d1 rows) and s2.
+bool encode_tmap_3d(CUtensorMap* tm, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1,
+                    uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2);
+
+// ---------------------------------------------------------------- GEMM
+enum GemmEpi : int {
+  EPI_BIAS_BF16 = ELASTO_EPI_BIAS_BF16,
+  EPI_BIAS_GELU_BF16 = ELASTO_EPI_BIAS_GELU_BF16,
+  EPI_BIAS_RESID_F32 = ELASTO_EPI_BIAS_RESID_F32,
+  EPI_BIAS_F32 = ELASTO_EPI_BIAS_F32,
+  EPI_BIAS_RELU_BF16 = ELASTO_EPI_BIAS_RELU_BF16,
+  EPI_BIAS_RESID_RELU_BF16 = ELASTO_EPI_BIAS_RESID_RELU_BF16,
+  EPI_PATCH_POS_F32 = 16,  // patch embedding: out row remapped past the class token, + position embedding
+};
+
+struct GemmArgs {
+  int M, N, K;
+  int bn;                 // N tile (multiple of 32, <= 256)
+  const float* bias;      // [N] or null
+  void* out;              // [*, ldo]
+  int ldo;
+  const bf16* resid;      // [M, ldr] (RESID_RELU)
+  int ldr;
+  int patches;            // PATCH: patches per image
+  int tokens;             // PATCH: tokens per image (patches + 1)
+  const float* pos;       // PATCH: [tokens, N]
+  int* status;
+};
+
+struct GemmPlan {
+  CUtensorMap tmA, tmB;
+  GemmArgs args;          // M here is the capacity the A map was encoded for
+  int epi = 0;
+  bool valid = false;
+};
+
+// Pick the N tile for an M x N problem.
+int gemm_pick_bn(int M, int N);
+// Build maps/arguments for out = epi(A[M_cap, K] W[N, K]^T). A and W must stay
+// allocated for the plan's life.
+elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
+                        void* out, int ldo, int epi, int* status);
+// Launch for the first M (<= M_cap) rows.
+cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s);
+cudaError_t gemm_init_attributes();
+
+// ---------------------------------------------------------------- attention
+struct AttnPlan {
+  CUtensorMap tmQ, tmKV;
+  const bf16* qkv;
+  bf16* out;
+  int n, n_pad, heads, batch_cap;
+  int* status;
+  bool valid = false;
+};
+elasto_status attn_plan(AttnPlan* p, const bf16* qkv, bf16* out, int batch_cap, int n, int heads, int* status);
+cudaError_t attn_launch(const AttnPlan& p, int batch, cudaStream_t s);
+cudaError_t attn_init_attributes();
+
+// ---------------------------------------------------------------- small kernels
+cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf16* y, int rows, int d,
+                             cudaStream_t s);
+cudaError_t softmax_launch(const float* x, float* y, int rows, int cols, cudaStream_t s);
+// images [B, H, W, C] (bf16 or fp32) -> A [B * np, P*P*C] bf16 in (ky, kx, c)
+// order; also writes the class-token rows X[b * n] = cls + pos[0].
+cudaError_t patchify_launch(const void* images, int img_dtype, int B, int H, int W, int C, int P, bf16* A,
+                            float* X, const float* cls, const float* pos, int d, cudaStream_t s);
+// logits[b, c] = LN(X[b * n, :]) . head_w[c, :] + head_b[c], all fp32.
+cudaError_t head_launch(const float* X, int B, int n, int d, const float* g, const float* b, const float* Wh,
+                        const float* bh, int C, float* logits, cudaStream_t s);
+// gathers for create-time packing
+cudaError_t gather_rows_bf16(const bf16* src, int cols, const int32_t* idx, int nidx, bf16* dst, cudaStream_t s);
+cudaError_t gather_cols_bf16(const bf16* src, int rows, int cols, const int32_t* idx, int nidx, bf16* dst,
+                             cudaStream_t s);
+cudaError_t gather_f32(const float* src, const int32_t* idx, int nidx, float* dst, cudaStream_t s);
+cudaError_t convert_to_bf16(const void* src, int src_dtype, size_t n, bf16* dst, cudaStream_t s);
+cudaError_t convert_to_f32(const void* src, int src_dtype, size_t n, float* dst, cudaStream_t s);
+
+}  // namespace elasto

@@ -1,0 +1,388 @@
+// Memory-bound kernels of the DN forward and create-time packing:
+//  - LayerNorm (pre-norm blocks and the class-token norm, Section 4.1 / 5.2):
+//    one warp per row, fp32 statistics, vector loads, warp-shuffle reductions;
+//  - row softmax (Eq. 3's softmax as a standalone op): one warp per row;
+//  - patch extraction for the patch projection (N = HW/P^2 patches, Section
+//    4.1) and the class-token rows of the residual stream;
+//  - class-token LayerNorm + linear classifier in fp32;
+//  - the index gathers that build each mode's packed weights (the structured
+//    masks of Eq. 4 and 6 applied as deletion), and dtype conversions.
+// Also: TMA map encoding, error strings, device facts.
+#include <stdarg.h>
+#include <stdio.h>
+
+#include <mutex>
+
+#include <cudaTypedefs.h>
+
+#include "common.h"
+#include "ptx.cuh"
+
+namespace elasto {
+
+// ---------------------------------------------------------------- errors
+namespace {
+thread_local std::string g_last_error;
+}
+void set_error(const std::string& msg) { g_last_error = msg; }
+void clear_error() { g_last_error.clear(); }
+const char* last_error_cstr() { return g_last_error.c_str(); }
+elasto_status cuda_fail(cudaError_t e, const char* what) {
+  set_error(std::string(what) + ": " + cudaGetErrorString(e));
+  return ELASTO_ERR_CUDA;
+}
+
+int num_sms() {
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (cached[dev] == 0) {
+    int v = 0;
+    if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess) cached[dev] = v;
+  }
+  return cached[dev];
+}
+
+// ---------------------------------------------------------------- TMA maps
+namespace {
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+}  // namespace
+
+bool encode_tmap_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_stride_bytes,
+                    uint32_t box_inner, uint32_t box_outer) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {row_stride_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_tmap_3d(CUtensorMap* tm, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1,
+                    uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2) {
+  auto enc = get_encode();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {d0, d1, d2};
+  cuuint64_t strides[2] = {s1, s2};
+  cuuint32_t box[3] = {b0, b1, b2};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// ---------------------------------------------------------------- LayerNorm
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+
+// One warp per row; each lane holds VEC float2 pairs (d = 64 * VEC).
+template <int VEC>
+__global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g,
+                                                        const float* __restrict__ b, bf16* __restrict__ y,
+                                                        int rows, float inv_d) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  constexpr int D = 64 * VEC;
+  const float2* xr = reinterpret_cast<const float2*>(x + static_cast<size_t>(row) * D);
+  float2 v[VEC];
+  float s = 0.0f;
+#pragma unroll
+  for (int i = 0; i < VEC; ++i) {
+    v[i] = xr[i * 32 + lane];
+    s += v[i].x + v[i].y;
+  }
+  const float mean = warp_sum(s) * inv_d;
+  float ss = 0.0f;
+#pragma unroll
+  for (int i = 0; i < VEC; ++i) {
+    const float a = v[i].x - mean, c = v[i].y - mean;
+    ss += a * a + c * c;
+  }
+  const float rstd = rsqrtf(warp_sum(ss) * inv_d + 1e-6f);
+  const float2* g2 = reinterpret_cast<const float2*>(g);
+  const float2* b2 = reinterpret_cast<const float2*>(b);
+  uint32_t* yr = reinterpret_cast<uint32_t*>(y + static_cast<size_t>(row) * D);
+#pragma unroll
+  for (int i = 0; i < VEC; ++i) {
+    const float2 gg = g2[i * 32 + lane], bb = b2[i * 32 + lane];
+    yr[i * 32 + lane] = pack_bf16x2((v[i].x - mean) * rstd * gg.x + bb.x, (v[i].y - mean) * rstd * gg.y + bb.y);
+  }
+}
+
+__global__ void __launch_bounds__(256) softmax_kernel(const float* __restrict__ x, float* __restrict__ y, int rows,
+                                                      int cols) {
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (row >= rows) return;
+  const float* xr = x + static_cast<size_t>(row) * cols;
+  float* yr = y + static_cast<size_t>(row) * cols;
+  float m = -INFINITY;
+  for (int c = lane; c < cols; c += 32) m = fmaxf(m, xr[c]);
+  m = warp_max(m);
+  float s = 0.0f;
+  for (int c = lane; c < cols; c += 32) s += expf(xr[c] - m);
+  s = warp_sum(s);
+  const float inv = 1.0f / s;
+  for (int c = lane; c < cols; c += 32) yr[c] = expf(xr[c] - m) * inv;
+}
+
+}  // namespace
+
+cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf16* y, int rows, int d,
+                             cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  const dim3 grid((rows + 7) / 8);
+  const float inv_d = 1.0f / static_cast<float>(d);
+  switch (d / 64) {
+#define LN_CASE(V) \
+  case V: layernorm_kernel<V><<<grid, 256, 0, s>>>(x, g, b, y, rows, inv_d); break;
+    LN_CASE(1) LN_CASE(2) LN_CASE(3) LN_CASE(4) LN_CASE(5) LN_CASE(6) LN_CASE(8) LN_CASE(10) LN_CASE(12)
+    LN_CASE(16)
+#undef LN_CASE
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t softmax_launch(const float* x, float* y, int rows, int cols, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  softmax_kernel<<<(rows + 7) / 8, 256, 0, s>>>(x, y, rows, cols);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- patches
+namespace {
+
+// One thread per 2 output elements of A[B * np, P*P*C] ((ky, kx, c) order);
+// the class-token rows are written by the first B * d threads.
+template <typename T>
+__global__ void patchify_kernel(const T* __restrict__ img, int B, int H, int W, int C, int P, bf16* __restrict__ A,
+                                float* __restrict__ X, const float* __restrict__ cls, const float* __restrict__ pos,
+                                int d) {
+  const int gw = W / P, np = (H / P) * gw, K = P * P * C;
+  const size_t total2 = static_cast<size_t>(B) * np * K / 2;
+  const size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (t < static_cast<size_t>(B) * d) {
+    const int bb = static_cast<int>(t / d), c = static_cast<int>(t % d);
+    X[static_cast<size_t>(bb) * (np + 1) * d + c] = cls[c] + pos[c];
+  }
+  if (t >= total2) return;
+  float v[2];
+#pragma unroll
+  for (int e = 0; e < 2; ++e) {
+    const size_t idx = 2 * t + e;
+    const int k = static_cast<int>(idx % K);
+    const size_t row = idx / K;
+    const int p = static_cast<int>(row % np), bb = static_cast<int>(row / np);
+    const int c = k % C, kx = (k / C) % P, ky = k / (C * P);
+    const int yy = (p / gw) * P + ky, xx = (p % gw) * P + kx;
+    const T val = img[((static_cast<size_t>(bb) * H + yy) * W + xx) * C + c];
+    if constexpr (sizeof(T) == 2)
+      v[e] = __bfloat162float(val);
+    else
+      v[e] = static_cast<float>(val);
+  }
+  reinterpret_cast<uint32_t*>(A)[t] = pack_bf16x2(v[0], v[1]);
+}
+
+}  // namespace
+
+cudaError_t patchify_launch(const void* images, int img_dtype, int B, int H, int W, int C, int P, bf16* A, float* X,
+                            const float* cls, const float* pos, int d, cudaStream_t s) {
+  const size_t total2 = static_cast<size_t>(B) * (H / P) * (W / P) * P * P * C / 2;
+  const size_t threads = total2 > static_cast<size_t>(B) * d ? total2 : static_cast<size_t>(B) * d;
+  const unsigned blocks = static_cast<unsigned>((threads + 255) / 256);
+  if (img_dtype == ELASTO_BF16)
+    patchify_kernel<bf16><<<blocks, 256, 0, s>>>(static_cast<const bf16*>(images), B, H, W, C, P, A, X, cls, pos, d);
+  else
+    patchify_kernel<float><<<blocks, 256, 0, s>>>(static_cast<const float*>(images), B, H, W, C, P, A, X, cls, pos,
+                                                  d);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- classifier
+namespace {
+
+constexpr int HEAD_IMGS = 8;     // class-token rows per CTA
+constexpr int HEAD_CLASSES = 64; // classes per CTA
+
+// grid (ceil(B / 8), ceil(C / 64)), 256 threads: LayerNorm of up to 8 class
+// tokens into shared memory (fp32), then each warp computes 8 classes x 8
+// images of dot products with float4 loads of the classifier rows.
+__global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, int B, int n, int d,
+                                                   const float* __restrict__ g, const float* __restrict__ bta,
+                                                   const float* __restrict__ Wh, const float* __restrict__ bh, int C,
+                                                   float* __restrict__ logits) {
+  extern __shared__ float sy[];  // [HEAD_IMGS][d]
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int b0 = blockIdx.x * HEAD_IMGS;
+  const int nimg = min(HEAD_IMGS, B - b0);
+  if (warp < nimg) {
+    const float* xr = X + static_cast<size_t>(b0 + warp) * n * d;  // class token row
+    float s = 0.0f;
+    for (int c = lane; c < d; c += 32) s += xr[c];
+    const float mean = warp_sum(s) / d;
+    float ss = 0.0f;
+    for (int c = lane; c < d; c += 32) {
+      const float a = xr[c] - mean;
+      ss += a * a;
+    }
+    const float rstd = rsqrtf(warp_sum(ss) / d + 1e-6f);
+    for (int c = lane; c < d; c += 32) sy[warp * d + c] = (xr[c] - mean) * rstd * g[c] + bta[c];
+  }
+  __syncthreads();
+  const int c0 = blockIdx.y * HEAD_CLASSES;
+  for (int cc = warp; cc < HEAD_CLASSES; cc += 8) {
+    const int cls = c0 + cc;
+    if (cls >= C) break;
+    const float* wr = Wh + static_cast<size_t>(cls) * d;
+    float acc[HEAD_IMGS];
+#pragma unroll
+    for (int i = 0; i < HEAD_IMGS; ++i) acc[i] = 0.0f;
+    for (int c = lane * 4; c < d; c += 128) {
+      const float4 wv = *reinterpret_cast<const float4*>(wr + c);
+#pragma unroll
+      for (int i = 0; i < HEAD_IMGS; ++i) {
+        if (i < nimg) {
+          const float4 yv = *reinterpret_cast<const float4*>(sy + i * d + c);
+          acc[i] += wv.x * yv.x + wv.y * yv.y + wv.z * yv.z + wv.w * yv.w;
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < HEAD_IMGS; ++i) {
+      const float v = warp_sum(acc[i]);
+      if (lane == 0 && i < nimg) logits[static_cast<size_t>(b0 + i) * C + cls] = v + bh[cls];
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t head_launch(const float* X, int B, int n, int d, const float* g, const float* b, const float* Wh,
+                        const float* bh, int C, float* logits, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  dim3 grid((B + HEAD_IMGS - 1) / HEAD_IMGS, (C + HEAD_CLASSES - 1) / HEAD_CLASSES);
+  head_kernel<<<grid, 256, HEAD_IMGS * d * sizeof(float), s>>>(X, B, n, d, g, b, Wh, bh, C, logits);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- packing
+namespace {
+
+__global__ void gather_rows_kernel(const bf16* __restrict__ src, int cols, const int32_t* __restrict__ idx,
+                                   int nidx, bf16* __restrict__ dst) {
+  const size_t total = static_cast<size_t>(nidx) * cols;
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const size_t r = t / cols, c = t % cols;
+    dst[t] = src[static_cast<size_t>(idx[r]) * cols + c];
+  }
+}
+
+__global__ void gather_cols_kernel(const bf16* __restrict__ src, int rows, int cols, const int32_t* __restrict__ idx,
+                                   int nidx, bf16* __restrict__ dst) {
+  const size_t total = static_cast<size_t>(rows) * nidx;
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const size_t r = t / nidx, c = t % nidx;
+    const int32_t k = idx[c];
+    dst[t] = k >= 0 ? src[r * cols + k] : __float2bfloat16_rn(0.0f);
+  }
+}
+
+__global__ void gather_f32_kernel(const float* __restrict__ src, const int32_t* __restrict__ idx, int nidx,
+                                  float* __restrict__ dst) {
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t < nidx) dst[t] = src[idx[t]];
+}
+
+template <typename T>
+__global__ void to_bf16_kernel(const T* __restrict__ src, size_t n, bf16* __restrict__ dst) {
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < n;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    if constexpr (sizeof(T) == 2)
+      dst[t] = src[t];
+    else
+      dst[t] = __float2bfloat16_rn(src[t]);
+  }
+}
+
+template <typename T>
+__global__ void to_f32_kernel(const T* __restrict__ src, size_t n, float* __restrict__ dst) {
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < n;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    if constexpr (sizeof(T) == 2)
+      dst[t] = __bfloat162float(src[t]);
+    else
+      dst[t] = src[t];
+  }
+}
+
+unsigned grid_for(size_t n) {
+  const size_t b = (n + 255) / 256;
+  return static_cast<unsigned>(b < 65536 ? (b > 0 ? b : 1) : 65536);
+}
+
+}  // namespace
+
+cudaError_t gather_rows_bf16(const bf16* src, int cols, const int32_t* idx, int nidx, bf16* dst, cudaStream_t s) {
+  if (nidx <= 0 || cols <= 0) return cudaSuccess;
+  gather_rows_kernel<<<grid_for(static_cast<size_t>(nidx) * cols), 256, 0, s>>>(src, cols, idx, nidx, dst);
+  return cudaGetLastError();
+}
+cudaError_t gather_cols_bf16(const bf16* src, int rows, int cols, const int32_t* idx, int nidx, bf16* dst,
+                             cudaStream_t s) {
+  if (nidx <= 0 || rows <= 0) return cudaSuccess;
+  gather_cols_kernel<<<grid_for(static_cast<size_t>(rows) * nidx), 256, 0, s>>>(src, rows, cols, idx, nidx, dst);
+  return cudaGetLastError();
+}
+cudaError_t gather_f32(const float* src, const int32_t* idx, int nidx, float* dst, cudaStream_t s) {
+  if (nidx <= 0) return cudaSuccess;
+  gather_f32_kernel<<<(nidx + 255) / 256, 256, 0, s>>>(src, idx, nidx, dst);
+  return cudaGetLastError();
+}
+cudaError_t convert_to_bf16(const void* src, int src_dtype, size_t n, bf16* dst, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  if (src_dtype == ELASTO_BF16)
+    to_bf16_kernel<bf16><<<grid_for(n), 256, 0, s>>>(static_cast<const bf16*>(src), n, dst);
+  else
+    to_bf16_kernel<float><<<grid_for(n), 256, 0, s>>>(static_cast<const float*>(src), n, dst);
+  return cudaGetLastError();
+}
+cudaError_t convert_to_f32(const void* src, int src_dtype, size_t n, float* dst, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  if (src_dtype == ELASTO_BF16)
+    to_f32_kernel<bf16><<<grid_for(n), 256, 0, s>>>(static_cast<const bf16*>(src), n, dst);
+  else
+    to_f32_kernel<float><<<grid_for(n), 256, 0, s>>>(static_cast<const float*>(src), n, dst);
+  return cudaGetLastError();
+}
+
+}  // namespace elasto

@@ -1,0 +1,73 @@
+// Stateless kernel-level entry points (elasto_ops.h): each DN forward step on
+// its own, so every kernel can be checked against the fp64 definition of that
+// step at arbitrary (odd, ragged) shapes.
+#include "common.h"
+#include "elasto_internal.h"
+
+using namespace elasto;
+
+extern "C" {
+
+elasto_status elasto_op_gemm(void* stream, const void* A, const void* W, const float* bias, void* out,
+                             const void* resid, int M, int N, int K, int epilogue, int* status_device) {
+  clear_error();
+  if (!out || M <= 0 || N <= 0 || K < 0 || (K > 0 && (!A || !W)) || epilogue < 0 || epilogue > 5 ||
+      (epilogue == ELASTO_EPI_BIAS_RESID_RELU_BF16 && !resid)) {
+    set_error("elasto_op_gemm: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  elasto_status st = check_device();
+  if (st != ELASTO_OK) return st;
+  GemmPlan p;
+  st = gemm_plan(&p, static_cast<const bf16*>(A), M, static_cast<const bf16*>(W), N, K, bias, out, N, epilogue,
+                 status_device);
+  if (st != ELASTO_OK) return st;
+  p.args.resid = static_cast<const bf16*>(resid);
+  p.args.ldr = N;
+  ELASTO_CUDA_TRY(gemm_launch(p, M, static_cast<cudaStream_t>(stream)));
+  return ELASTO_OK;
+}
+
+elasto_status elasto_op_layernorm(void* stream, const float* x, const float* gamma, const float* beta, void* y,
+                                  int rows, int d) {
+  clear_error();
+  if (!x || !gamma || !beta || !y || rows <= 0 || d <= 0) {
+    set_error("elasto_op_layernorm: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int v = d / 64;
+  if (d % 64 != 0 || !(v <= 6 || v == 8 || v == 10 || v == 12 || v == 16)) {
+    set_error("elasto_op_layernorm: d must be 64 x {1..6, 8, 10, 12, 16}");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  ELASTO_CUDA_TRY(layernorm_launch(x, gamma, beta, static_cast<bf16*>(y), rows, d, static_cast<cudaStream_t>(stream)));
+  return ELASTO_OK;
+}
+
+elasto_status elasto_op_softmax(void* stream, const float* x, float* y, int rows, int cols) {
+  clear_error();
+  if (!x || !y || rows <= 0 || cols <= 0) {
+    set_error("elasto_op_softmax: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  ELASTO_CUDA_TRY(softmax_launch(x, y, rows, cols, static_cast<cudaStream_t>(stream)));
+  return ELASTO_OK;
+}
+
+elasto_status elasto_op_attention(void* stream, const void* qkv, void* out, int batch, int n, int heads,
+                                  int* status_device) {
+  clear_error();
+  if (!qkv || !out || batch <= 0 || n <= 0 || heads <= 0) {
+    set_error("elasto_op_attention: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  elasto_status st = check_device();
+  if (st != ELASTO_OK) return st;
+  AttnPlan p;
+  st = attn_plan(&p, static_cast<const bf16*>(qkv), static_cast<bf16*>(out), batch, n, heads, status_device);
+  if (st != ELASTO_OK) return st;
+  ELASTO_CUDA_TRY(attn_launch(p, batch, static_cast<cudaStream_t>(stream)));
+  return ELASTO_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,161 @@
+"""Each CUDA kernel on its own, through the C-ABI op entry points, against
+the fp64 oracle's matching sub-step, at odd and ragged shapes."""
+import numpy as np
+import pytest
+
+from helpers import bf16_to_f64, dev, empty_dev, stream_handle
+from oracle import vit as ov
+from paper_2609_10018_gb300 import binding, synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _bf16(rng, shape, scale=1.0):
+    return synth.f32_to_bf16_bits(rng.standard_normal(shape, dtype=np.float32) * np.float32(scale))
+
+
+def _status():
+    import torch
+    return torch.zeros(1, dtype=torch.int32, device="cuda")
+
+
+GEMM_CASES = [
+    # M, N, K, epilogue
+    (128, 256, 64, binding.EPI_BIAS_BF16),            # one tile
+    (200, 576, 384, binding.EPI_BIAS_BF16),           # ragged M, 3-head QKV width
+    (1000, 192, 48, binding.EPI_BIAS_BF16),           # K below one k-block (tiny patch projection)
+    (333, 1000, 768, binding.EPI_BIAS_F32),           # N not a multiple of 32 (classifier width)
+    (1537, 3072, 768, binding.EPI_BIAS_GELU_BF16),    # FC1
+    (1537, 768, 3072, binding.EPI_BIAS_RESID_F32),    # FC2 with residual
+    (257, 768, 0, binding.EPI_BIAS_RESID_F32),        # no kept channel: residual += bias
+    (6304, 2304, 768, binding.EPI_BIAS_BF16),         # ViT-B QKV at batch 32
+    (130, 200, 136, binding.EPI_BIAS_RELU_BF16),      # conv-like K
+    (130, 64, 72, binding.EPI_BIAS_RESID_RELU_BF16),
+    (64, 1152, 384, binding.EPI_BIAS_GELU_BF16),      # ViT-S 75 % MLP, M below one tile
+]
+
+
+@pytest.mark.parametrize("M,N,K,epi", GEMM_CASES)
+def test_gemm_epilogues_match_fp64(M, N, K, epi):
+    import torch
+    rng = np.random.default_rng(M * 7 + N * 3 + K)
+    A = _bf16(rng, (M, max(K, 8)))[:, :K].copy() if K else np.zeros((M, 0), np.uint16)
+    W = _bf16(rng, (N, max(K, 8)), 0.05)[:, :K].copy() if K else np.zeros((N, 0), np.uint16)
+    bias = rng.standard_normal(N).astype(np.float32)
+    ref = bf16_to_f64(A) @ bf16_to_f64(W).T + bias
+    f32_out = epi in (binding.EPI_BIAS_F32, binding.EPI_BIAS_RESID_F32)
+    resid = None
+    if epi == binding.EPI_BIAS_RESID_F32:
+        x0 = rng.standard_normal((M, N)).astype(np.float32)
+        out = dev(x0)
+        ref = ref + x0
+    else:
+        out = empty_dev((M, N), torch.float32 if f32_out else torch.uint16)
+    if epi == binding.EPI_BIAS_GELU_BF16:
+        ref = ov.gelu(ref)
+    elif epi == binding.EPI_BIAS_RELU_BF16:
+        ref = np.maximum(ref, 0)
+    elif epi == binding.EPI_BIAS_RESID_RELU_BF16:
+        r = _bf16(rng, (M, N))
+        resid = dev(r)
+        ref = np.maximum(ref + bf16_to_f64(r), 0)
+    st = _status()
+    dA = dev(A) if K else None
+    dW = dev(W) if K else None
+    db = dev(bias)
+    binding.elasto_op_gemm(stream_handle(), dA.data_ptr() if K else None, dW.data_ptr() if K else None,
+                           db.data_ptr(), out.data_ptr(), resid.data_ptr() if resid is not None else None,
+                           M, N, K, epi, st.data_ptr())
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    got = out.cpu().numpy().astype(np.float64) if f32_out else bf16_to_f64(out)
+    scale = float(np.max(np.abs(ref)))
+    if f32_out:
+        assert np.all(np.abs(got - ref) <= 1e-5 * scale + 1e-6 * np.abs(ref)), float(np.max(np.abs(got - ref)))
+    else:  # one bf16 rounding of the fp32 result
+        assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5 * scale), float(np.max(np.abs(got - ref)))
+
+
+def test_gemm_full_size_outproj_sampled_rows():
+    """ViT-B out-projection at batch 256 (M = 50432 = 394 tiles), sampled rows."""
+    import torch
+    M, N, K = 256 * 197, 768, 768
+    rng = np.random.default_rng(11)
+    A = _bf16(rng, (M, K))
+    W = _bf16(rng, (N, K), 0.03)
+    bias = rng.standard_normal(N).astype(np.float32)
+    x0 = rng.standard_normal((M, N)).astype(np.float32)
+    out = dev(x0)
+    binding.elasto_op_gemm(stream_handle(), dev(A).data_ptr(), dev(W).data_ptr(), dev(bias).data_ptr(),
+                           out.data_ptr(), None, M, N, K, binding.EPI_BIAS_RESID_F32, 0)
+    torch.cuda.synchronize()
+    rows = np.concatenate([np.arange(0, 130), rng.choice(M, 300, replace=False), np.arange(M - 130, M)])
+    got = out.cpu().numpy()[rows].astype(np.float64)
+    ref = bf16_to_f64(A[rows]) @ bf16_to_f64(W).T + bias + x0[rows]
+    assert np.max(np.abs(got - ref)) <= 1e-5 * np.max(np.abs(ref))
+
+
+@pytest.mark.parametrize("rows,d", [(1000, 192), (333, 384), (2051, 768), (7, 1024)])
+def test_layernorm_matches_fp64(rows, d):
+    import torch
+    rng = np.random.default_rng(rows + d)
+    x = (rng.standard_normal((rows, d)) * 2.0 + 0.7).astype(np.float32)
+    g = (1 + 0.1 * rng.standard_normal(d)).astype(np.float32)
+    b = (0.1 * rng.standard_normal(d)).astype(np.float32)
+    y = empty_dev((rows, d), torch.uint16)
+    binding.elasto_op_layernorm(stream_handle(), dev(x).data_ptr(), dev(g).data_ptr(), dev(b).data_ptr(),
+                                y.data_ptr(), rows, d)
+    torch.cuda.synchronize()
+    ref = ov.layer_norm(x.astype(np.float64), g, b)
+    got = bf16_to_f64(y)
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5 * np.max(np.abs(ref)))
+
+
+@pytest.mark.parametrize("rows,cols", [(100, 1), (64, 10), (300, 197), (17, 1000)])
+def test_softmax_matches_fp64(rows, cols):
+    import torch
+    rng = np.random.default_rng(rows * cols)
+    x = (rng.standard_normal((rows, cols)) * 4).astype(np.float32)
+    y = empty_dev((rows, cols), torch.float32)
+    binding.elasto_op_softmax(stream_handle(), dev(x).data_ptr(), y.data_ptr(), rows, cols)
+    torch.cuda.synchronize()
+    ref = ov.softmax_rows(x.astype(np.float64))
+    got = y.cpu().numpy().astype(np.float64)
+    assert np.max(np.abs(got - ref)) <= 1e-6
+    assert np.allclose(got.sum(1), 1.0, atol=1e-5)
+
+
+ATTN_CASES = [(2, 197, 3), (3, 65, 2), (1, 256, 1), (2, 1, 1), (2, 17, 4), (1, 129, 12)]
+
+
+@pytest.mark.parametrize("B,n,h", ATTN_CASES)
+def test_attention_matches_fp64(B, n, h):
+    import torch
+    rng = np.random.default_rng(B * 1000 + n * 10 + h)
+    qkv = _bf16(rng, (B, n, 3, h, 64))
+    out = empty_dev((B, n, h * 64), torch.uint16)
+    st = _status()
+    binding.elasto_op_attention(stream_handle(), dev(qkv).data_ptr(), out.data_ptr(), B, n, h, st.data_ptr())
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    q = bf16_to_f64(qkv)
+    ref = np.concatenate([ov.attention(q[:, :, 0, j], q[:, :, 1, j], q[:, :, 2, j], 64) for j in range(h)], axis=-1)
+    got = bf16_to_f64(out)
+    # P is rounded to bf16 before P.V and O to bf16 at the end
+    assert np.max(np.abs(got - ref)) <= 1e-2 * np.max(np.abs(ref)), float(np.max(np.abs(got - ref)))
+
+
+def test_attention_full_size_sampled():
+    """ViT-B shape at batch 256: 256 x 12 heads x 197 tokens; sampled images."""
+    import torch
+    B, n, h = 256, 197, 12
+    rng = np.random.default_rng(5)
+    qkv = _bf16(rng, (B, n, 3, h, 64))
+    out = empty_dev((B, n, h * 64), torch.uint16)
+    binding.elasto_op_attention(stream_handle(), dev(qkv).data_ptr(), out.data_ptr(), B, n, h, 0)
+    torch.cuda.synchronize()
+    got = bf16_to_f64(out)
+    for b in (0, 1, 128, 255):
+        q = bf16_to_f64(qkv[b])
+        ref = np.concatenate([ov.attention(q[:, 0, j], q[:, 1, j], q[:, 2, j], 64) for j in range(h)], axis=-1)
+        assert np.max(np.abs(got[b] - ref)) <= 1e-2 * np.max(np.abs(ref))

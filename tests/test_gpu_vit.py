@@ -1,0 +1,174 @@
+"""End-to-end DN forward of the elastic ViTs through the C-ABI against the
+fp64 oracle: every mode of the tiny, ViT-S/16 and ViT-B/16 configurations,
+bit-exact packed layouts, mode switching, degenerate tables.
+
+Acceptance (per mode): max|dlogit| <= 1e-2 * max|logit_oracle|, and top-1
+agreement >= 99.9 % where the image count makes that meaningful (2000 tiny
+images per mode); at ViT-S/B sizes the oracle checks sampled images."""
+import numpy as np
+import pytest
+
+from helpers import dev, empty_dev, margin, rel_err, stream_handle, top1_agreement
+from oracle import vit as ov
+from paper_2609_10018_gb300 import binding, synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-2
+
+
+def _run(model, images_dev, batch, classes, mode):
+    import torch
+    logits = empty_dev((batch, classes), torch.float32)
+    model.set_mode(mode)
+    model.forward(stream_handle(), images_dev.data_ptr(), batch, logits.data_ptr())
+    model.sync_status(stream_handle())
+    return logits.cpu().numpy().astype(np.float64)
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    cfg = synth.TINY
+    w = synth.make_vit_weights(cfg)
+    tables = synth.make_vit_tables(cfg)
+    return cfg, w, ov.widen_all(w), tables
+
+
+def test_tiny_all_modes_2000_images(tiny):
+    cfg, w, wide, tables = tiny
+    n_img = 2000
+    img = synth.make_images(cfg, n_img)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=n_img) as model:
+        x = dev(img)
+        for m, t in enumerate(tables):
+            got = _run(model, x, n_img, cfg.classes, m)
+            ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img)
+            err, agree = rel_err(got, ref), top1_agreement(got, ref)
+            mg = margin(ref)
+            print(f"tiny mode {m}: err {err:.2e} top1 {agree:.4f} margin p1/p50 {np.percentile(mg, 1):.3e}/"
+                  f"{np.median(mg):.3e}")
+            assert err <= TOL
+            assert agree >= 0.999
+
+
+def test_tiny_batch_8_matches_oracle(tiny):
+    cfg, w, wide, tables = tiny
+    img = synth.make_images(cfg, cfg.batch)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=cfg.batch) as model:
+        x = dev(img)
+        for m, t in enumerate(tables):
+            assert rel_err(_run(model, x, cfg.batch, cfg.classes, m),
+                           ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img)) <= TOL
+
+
+@pytest.mark.parametrize("cfg", [synth.TINY, synth.VIT_S, synth.VIT_B], ids=lambda c: c.name)
+def test_packed_layouts_bit_exact(cfg):
+    w = synth.make_vit_weights(cfg)
+    tables = synth.make_vit_tables(cfg)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=1) as model:
+        for m, t in enumerate(tables):
+            for l in range(cfg.layers):
+                ref = ov.vit_pack_layer(w, cfg, l, t["heads"][l], t["mlp"][l])
+                for which, name in enumerate(ov.PACK_ORDER):
+                    out = np.empty_like(ref[name])
+                    model.export_packed(m, l, which, out)
+                    assert out.tobytes() == ref[name].tobytes(), (m, l, name)
+
+
+def _sampled_parity(cfg, batch, sample, modes=None):
+    w = synth.make_vit_weights(cfg)
+    wide = ov.widen_all(w)
+    tables = synth.make_vit_tables(cfg)
+    img = synth.make_images(cfg, batch)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=batch) as model:
+        x = dev(img)
+        for m in (modes if modes is not None else range(len(tables))):
+            t = tables[m]
+            got = _run(model, x, batch, cfg.classes, m)
+            ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img[sample])
+            err = rel_err(got[sample], ref)
+            print(f"{cfg.name} B={batch} mode {m}: err {err:.2e}, top-1 {top1_agreement(got[sample], ref):.3f}")
+            assert err <= TOL
+            assert top1_agreement(got[sample], ref) == 1.0 or np.min(margin(ref)) < 2 * TOL * np.max(np.abs(ref))
+            assert np.all(np.isfinite(got))
+
+
+def test_vit_s_batch_64_all_modes():
+    _sampled_parity(synth.VIT_S, 64, np.array([0, 1, 31, 62, 63]))
+
+
+def test_vit_b_batch_256_all_modes():
+    _sampled_parity(synth.VIT_B, 256, np.array([0, 97, 254, 255]))
+
+
+@pytest.mark.parametrize("batch", [1, 32])
+def test_vit_b_small_batches(batch):
+    _sampled_parity(synth.VIT_B, batch, np.array([0, batch - 1]), modes=[0, 4])
+
+
+def test_mode_switch_between_enqueued_forwards(tiny):
+    """set_mode only affects forwards enqueued after it; no sync in between."""
+    import torch
+    cfg, w, wide, tables = tiny
+    img = synth.make_images(cfg, cfg.batch)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=cfg.batch) as model:
+        x = dev(img)
+        outs = [empty_dev((cfg.batch, cfg.classes), torch.float32) for _ in range(4)]
+        seq = [1, 0, 1, 1]
+        s = stream_handle()
+        for o, m in zip(outs, seq):
+            model.set_mode(m)
+            model.forward(s, x.data_ptr(), cfg.batch, o.data_ptr())
+        model.sync_status(s)
+        for o, m in zip(outs, seq):
+            t = tables[m]
+            assert rel_err(o.cpu().numpy().astype(np.float64),
+                           ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img)) <= TOL
+        assert model.mode == 1
+
+
+def test_forward_host_equals_device_forward(tiny):
+    cfg, w, wide, tables = tiny
+    img = synth.make_images(cfg, 5)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=8) as model:
+        dev_out = _run(model, dev(img), 5, cfg.classes, 1)
+        host_out = np.zeros((5, cfg.classes), np.float32)
+        model.forward_host(img, host_out)
+        assert np.array_equal(host_out.astype(np.float64), dev_out)
+
+
+def test_degenerate_and_non_nested_tables():
+    """Layers keeping no head and/or no MLP channel, a channel count that is
+    not a multiple of 8, and tables that are not nested across modes."""
+    cfg = synth.vit_small_variant(synth.TINY, dtype=synth.BF16)
+    w = synth.make_vit_weights(cfg)
+    wide = ov.widen_all(w)
+    t0 = synth.make_vit_tables(cfg)[0]
+    rng = np.random.default_rng(3)
+    odd = {"heads": [np.sort(rng.choice(3, k, replace=False)).astype(np.int32) for k in (0, 1, 3, 2, 0, 1)],
+           "mlp": [np.sort(rng.choice(768, k, replace=False)).astype(np.int32) for k in (100, 0, 768, 1, 0, 37)]}
+    tables = [t0, odd] + synth.make_vit_tables(cfg, nested=False)[1:]
+    img = synth.make_images(cfg, 6)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=6) as model:
+        x = dev(img)
+        for m, t in enumerate(tables):
+            got = _run(model, x, 6, cfg.classes, m)
+            ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img)
+            assert rel_err(got, ref) <= TOL, m
+
+
+def test_batch_limits_and_bad_mode(tiny):
+    cfg, w, wide, tables = tiny
+    import torch
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=4) as model:
+        x = dev(synth.make_images(cfg, 5))
+        y = empty_dev((5, cfg.classes), torch.float32)
+        with pytest.raises(binding.ElastoError) as e:
+            model.forward(stream_handle(), x.data_ptr(), 5, y.data_ptr())
+        assert e.value.status == binding.ERR_INVALID_ARG
+        with pytest.raises(binding.ElastoError) as e:
+            model.set_mode(2)
+        assert e.value.status == binding.ERR_BAD_MODE
+        assert model.mode == 0
+        assert model.query(binding.Q_N_MODES) == 2
+        assert model.query(binding.Q_PACKED_BYTES, 1) < model.query(binding.Q_PACKED_BYTES, 0)
