@@ -1,0 +1,447 @@
+#!/usr/bin/env python3
+"""Benchmark of the elastic ViT-B/16 descendant-network forward on GB300.
+
+Headline workload: ViT-B/16 (224x224, 197 tokens, d 768, 12 heads, MLP 3072,
+1000 classes), full mode, batch 256, bf16 weights/activations with fp32
+accumulation, synthetic seeded weights and images. One step = one forward
+of one batch. Reported with it, in the same JSON line: images/s and % of the
+dense BF16 peak for every mode at batch 256, batch-1 latency per mode (CUDA
+graph replay), mode-switch cost, the dominant kernel's roofline measured live
+with CUDA events, the end-to-end number through host buffers, the fp64
+oracle timed on the host cores, and the SM clocks seen during timing.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl elasto|reference]
+
+Multi-GPU (torchrun): each rank runs an independent replica on its own
+batch (the path has no exchange step); value = all ranks' images / max time.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "images/sec per mode on 1 GB300 (BF16) and % of dense BF16 tensor peak; mode-switch µs"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+L2_FLUSH_BYTES = 256 << 20
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=10)
+    p.add_argument("--impl", choices=["elasto", "reference"], default="elasto")
+    p.add_argument("--batch", type=int, default=256)
+    p.add_argument("--mode", type=int, default=0)
+    p.add_argument("--quick", action="store_true", help="headline only: skip per-mode sweep, latency, baseline")
+    return p.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            pk = json.load(f)
+        return {k: float(pk[k]) for k in FALLBACK_PEAKS}, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while timing."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100", "-f", self.path],
+                                         stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.2)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path).read().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 9:
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        smax = [num(r[2]) for r in rows if num(r[2]) is not None]
+        power = [num(r[3]) for r in rows if num(r[3]) is not None]
+        loaded = [s for s, p in zip(sm, power) if p is not None and p > 300] or sm
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(smax) if smax else None, "reasons": reasons, "samples": len(rows),
+                "power_w_max": max(power) if power else None}
+
+
+# ---------------------------------------------------------------------------- oracle timing
+def oracle_cpu_baseline(cfg, budget_s: float = 12.0, mode: int = 0):
+    """The fp64 oracle (as it stands) on the host cores: images/s of the DN
+    forward on a bounded sample of the same workload."""
+    from oracle import vit as ov
+    from paper_2609_10018_gb300 import synth
+    w = ov.widen_all(synth.make_vit_weights(cfg))
+    t = synth.make_vit_tables(cfg)[mode]
+    img = synth.make_images(cfg, 64)
+    t0 = time.perf_counter()
+    ov.vit_forward_sliced(w, cfg, t["heads"], t["mlp"], img[:1])
+    one = time.perf_counter() - t0
+    n = int(max(1, min(32, budget_s / max(one, 1e-3))))
+    t0 = time.perf_counter()
+    ov.vit_forward_sliced(w, cfg, t["heads"], t["mlp"], img[:n])
+    dt = time.perf_counter() - t0
+    cores = int(os.environ.get("OPENBLAS_NUM_THREADS", os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1)))
+    return {"value": n / dt, "unit": "images/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} images of the {cfg.name} full-mode forward in one fp64 oracle call "
+                      f"({dt:.1f} s; numpy/OpenBLAS on {cores} host threads)"}
+
+
+def run_reference(args):
+    """Reference arm: the fp64 oracle on the host cores, same metric and
+    workload, each step a bounded sample (1 image) of it."""
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    from oracle import vit as ov
+    from paper_2609_10018_gb300 import synth
+    cfg = synth.VIT_B
+    w = ov.widen_all(synth.make_vit_weights(cfg))
+    t = synth.make_vit_tables(cfg)[args.mode]
+    img = synth.make_images(cfg, args.warmup + args.steps)
+    for i in range(args.warmup):
+        ov.vit_forward_sliced(w, cfg, t["heads"], t["mlp"], img[i:i + 1])
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        ov.vit_forward_sliced(w, cfg, t["heads"], t["mlp"], img[args.warmup + i:args.warmup + i + 1])
+    dt = time.perf_counter() - t0
+    value = args.steps / dt
+    cores = int(os.environ.get("OPENBLAS_NUM_THREADS", os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1)))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded N(0,0.02) weights, U[0,1) pixels)",
+            "config": {"workload": f"elastic ViT-B/16 DN forward, mode {args.mode}, 1 image per step "
+                                   f"(bounded sample of the batch-{args.batch} workload)", "global_batch": 1,
+                       "seq_len": 197, "parallelism": "host cores"},
+            "cpu_baseline": {"value": value, "unit": "images/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{args.steps} timed single-image forwards after {args.warmup} warm-up"},
+            "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+# ---------------------------------------------------------------------------- profiles
+def committed_traffic(kernel: str, src_file: str):
+    """Per-launch DRAM traffic of `kernel` from a committed ncu summary, if
+    it was taken on the current kernel source (sha256 match), else None."""
+    sha = hashlib.sha256(open(src_file, "rb").read()).hexdigest()
+    pdir = os.path.join(ROOT, "profiles")
+    if not os.path.isdir(pdir):
+        return None
+    for f in sorted(os.listdir(pdir)):
+        if not f.endswith((".txt", ".md")):
+            continue
+        text = open(os.path.join(pdir, f)).read()
+        for m in re.finditer(r"traffic_kernel:\s*(\S+)\s+traffic_bytes_per_launch:\s*([0-9.eE+]+)\s+"
+                             r"source_sha256:\s*([0-9a-f]+)", text):
+            if m.group(1) == kernel and m.group(3) == sha:
+                return float(m.group(2))
+    return None
+
+
+GEMM_ROLES = ("qkv", "proj", "fc1", "fc2")
+
+
+def label_records(recs):
+    """Name each launch record: GEMMs by their role in the layer (the forward
+    launches QKV, out-proj, FC1, FC2 in that order; the patch projection is
+    outside the layers)."""
+    seen = {}
+    for r in recs:
+        if r["kind"] != "gemm":
+            yield r["kind"], r
+            continue
+        if r["layer"] < 0:
+            yield "gemm.patch", r
+            continue
+        i = seen.get(r["layer"], 0)
+        seen[r["layer"]] = i + 1
+        yield "gemm." + (GEMM_ROLES[i] if i < len(GEMM_ROLES) else "other"), r
+
+
+# ---------------------------------------------------------------------------- main bench
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    import torch
+    from paper_2609_10018_gb300 import binding, synth
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    peaks, peak_src = load_peaks()
+    cfg = synth.VIT_B
+    B = args.batch
+    weights = synth.make_vit_weights(cfg)
+    tables = synth.make_vit_tables(cfg)
+    model = binding.ElasticModel.vit(cfg, weights, tables, max_batch=B)
+    images_np = synth.make_images(cfg, B, seed=cfg.seeds[2] + rank)
+    images = torch.from_numpy(images_np).cuda()
+    logits = torch.empty(B, cfg.classes, dtype=torch.float32, device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+
+    def timed_steps(mode, steps, warmup, profile=True):
+        model.set_mode(mode)
+        model.profile(profile)
+        for _ in range(warmup):
+            model.forward(sh, images.data_ptr(), B, logits.data_ptr())
+        torch.cuda.synchronize()
+        times, per_kind, recs_first = [], {}, None
+        for _ in range(steps):
+            flush.fill_(1.0)  # > L2: every step starts cold
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            model.forward(sh, images.data_ptr(), B, logits.data_ptr())
+            e1.record(stream)
+            if profile:
+                recs = model.profile_read()
+                recs_first = recs_first or recs
+                for key, r in label_records(recs):
+                    for k in (key, "gemm") if key.startswith("gemm.") else (key,):
+                        acc = per_kind.setdefault(k, [0.0, 0.0, 0.0, 0])
+                        acc[0] += r["ms"]
+                        acc[1] += r["macs"]
+                        acc[2] += r["bytes"]
+                        acc[3] += 1
+            torch.cuda.synchronize()
+            times.append(e0.elapsed_time(e1))
+        model.profile(False)
+        return times, per_kind, recs_first
+
+    # ------------------------------------------------ headline: full mode, batch B
+    times, per_kind, recs = timed_steps(args.mode, 3, args.warmup)  # warm-up incl. profiler
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clk = ClockSampler(local)
+    clk.start()
+    times, per_kind, recs = timed_steps(args.mode, args.steps, 0)
+    clocks = clk.stop()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    total_ms = float(sum(times))
+    if dist:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = world * B * args.steps / (total_ms / 1e3)
+    macs_img = model.query(binding.Q_MODE_MACS, args.mode)
+    tflops = 2.0 * macs_img * B * args.steps / (float(sum(times)) / 1e3) / 1e12
+    launches = model.query(binding.Q_LAUNCHES, args.mode)
+
+    # dominant kernel: the tcgen05 GEMM (all its launches in the step)
+    total_kernel_ms = sum(v[0] for k, v in per_kind.items() if k != "gemm")
+    kinds = {}
+    for k, v in per_kind.items():
+        e = {"ms_per_step": v[0] / args.steps, "share": v[0] / total_kernel_ms,
+             "launches_per_step": v[3] / args.steps}
+        if v[1] > 0:
+            e["tflops"] = 2.0 * v[1] / (v[0] / 1e3) / 1e12
+        if k in ("layernorm", "attention", "patchify", "head"):
+            e["gbs"] = v[2] / (v[0] / 1e3) / 1e9
+        kinds[k] = e
+    g = per_kind.get("gemm", [1e-9, 0, 0, 1])
+    gemm_tflops = 2.0 * g[1] / (g[0] / 1e3) / 1e12
+    peak_t = peaks["bf16_tflops_sustained"]
+    traffic = committed_traffic("gemm_tc_kernel", os.path.join(ROOT, "paper_2609_10018_gb300", "csrc", "gemm.cu"))
+    roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (all epilogues; tcgen05 M=128 tiles)",
+                "achieved": gemm_tflops, "peak": peak_t, "unit": "TFLOP/s", "frac": gemm_tflops / peak_t,
+                "traffic": traffic, "peak_source": f"{peak_src} bf16_tflops_sustained (GEMMs timed inside a "
+                                                   f"{statistics.mean(times):.1f} ms step)",
+                "algorithmic": "2 x M x N x K per launch (kept widths only), summed over the step's GEMM launches",
+                "launches_per_step": g[3] / args.steps, "ms_per_step": g[0] / args.steps}
+
+    line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "data": "synthetic (seeded N(0,0.02) weights, U[0,1) pixels; ImageNet-shaped)",
+            "config": {"workload": f"elastic ViT-B/16 DN forward, mode {args.mode} "
+                                   f"({len(tables[args.mode]['heads'][0])} heads, MLP "
+                                   f"{len(tables[args.mode]['mlp'][0])}), batch {B}",
+                       "global_batch": B * world, "seq_len": cfg.tokens, "parallelism": f"replicas x{world}",
+                       "l2": "flushed between timed steps (256 MiB write)"},
+            "tflops": tflops, "frac_of_bf16_peak": tflops / peaks["bf16_tflops"],
+            "peaks": {**peaks, "source": peak_src}, "roofline": roofline, "kernels": kinds,
+            "gpu_launches": launches * args.steps, "clocks": clocks}
+
+    if rank == 0 and not args.quick:
+        line["per_mode"] = []
+        for m in range(len(tables)):
+            t_m, _, _ = timed_steps(m, 20, 3, profile=False)
+            ips = B * len(t_m) / (sum(t_m) / 1e3)
+            mm = model.query(binding.Q_MODE_MACS, m)
+            tf = 2.0 * mm * ips / 1e12
+            line["per_mode"].append({"mode": m, "heads": int(len(tables[m]["heads"][0])),
+                                     "mlp": int(len(tables[m]["mlp"][0])), "images_per_s": ips,
+                                     "tflops": tf, "frac_of_bf16_peak": tf / peaks["bf16_tflops"],
+                                     "gflop_per_image": 2 * mm / 1e9,
+                                     "packed_weight_mb": model.query(binding.Q_PACKED_BYTES, m) / 1e6})
+        line["latency"] = batch1_latency(model, cfg, tables, torch, binding, peaks)
+        line["mode_switch_us"] = mode_switch(model, cfg, tables, torch, binding)
+        line["e2e"] = e2e(model, cfg, images_np, B, args, torch, binding)
+        line["cpu_baseline"] = oracle_cpu_baseline(cfg)
+    elif rank == 0:
+        line["e2e"] = e2e(model, cfg, images_np, B, args, torch, binding)
+    model.close()
+    if rank == 0:
+        print(json.dumps(line))
+    if dist:
+        dist.destroy_process_group()
+
+
+def batch1_latency(model, cfg, tables, torch, binding, peaks):
+    """Per mode at batch 1 (the paper's latency protocol: 10 warm-up, 50
+    trials), CUDA-graph replay of the whole forward; weight bytes / latency."""
+    out = []
+    img = torch.from_numpy(__import__("paper_2609_10018_gb300.synth", fromlist=["x"]).make_images(cfg, 1)).cuda()
+    lg = torch.empty(1, cfg.classes, dtype=torch.float32, device="cuda")
+    for m in range(len(tables)):
+        model.set_mode(m)
+        side = torch.cuda.Stream()
+        with torch.cuda.stream(side):
+            model.forward(side.cuda_stream, img.data_ptr(), 1, lg.data_ptr())
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            model.forward(torch.cuda.current_stream().cuda_stream, img.data_ptr(), 1, lg.data_ptr())
+        for _ in range(10):
+            g.replay()
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(50):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            g.replay()
+            e1.record()
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        med = statistics.median(ts)
+        wbytes = model.query(binding.Q_PACKED_BYTES, m) + model.query(binding.Q_SHARED_BYTES)
+        out.append({"mode": m, "batch": 1, "us_p50": med * 1e3, "us_p99": float(np.percentile(ts, 99)) * 1e3,
+                    "weight_gbs": wbytes / (med / 1e3) / 1e9,
+                    "frac_of_hbm": wbytes / (med / 1e3) / 1e9 / peaks["hbm_gbs"]})
+        del g
+    return out
+
+
+def mode_switch(model, cfg, tables, torch, binding):
+    """(i) host cost of elasto_set_mode; (ii) device-visible cost: latency of
+    the first batch-1 forward after a switch minus the same mode's steady
+    state (eager launches)."""
+    import ctypes
+    lib = binding.lib()
+    h = ctypes.c_void_p(model.handle)
+    n = 100_000
+    t0 = time.perf_counter_ns()
+    for i in range(n):
+        lib.elasto_set_mode(h, i & 1)
+    host_us = (time.perf_counter_ns() - t0) / n / 1e3
+    img = torch.from_numpy(__import__("paper_2609_10018_gb300.synth", fromlist=["x"]).make_images(cfg, 1)).cuda()
+    lg = torch.empty(1, cfg.classes, dtype=torch.float32, device="cuda")
+    sh = torch.cuda.current_stream().cuda_stream
+    last = len(tables) - 1
+
+    def lat(mode):
+        model.set_mode(mode)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        model.forward(sh, img.data_ptr(), 1, lg.data_ptr())
+        e1.record()
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1)
+    for _ in range(5):
+        lat(0), lat(last)
+    switched = [lat(m) for _ in range(100) for m in (0, last)]
+    steady = [lat(m) for m in (0, last) for _ in range(100)]
+    return {"host_set_mode_us": host_us, "first_forward_after_switch_us": 1e3 * statistics.mean(switched),
+            "steady_forward_us": 1e3 * statistics.mean(steady),
+            "device_visible_switch_us": 1e3 * (statistics.mean(switched) - statistics.mean(steady)),
+            "protocol": f"batch 1, alternating modes 0 and {last}, 200 forwards each way, eager launches",
+            "paper_context": "about 50.4 ms on Jetson Orin (Section 6.2)"}
+
+
+def e2e(model, cfg, images_np, B, args, torch, binding):
+    """Same metric through the public host-buffer call: every step copies the
+    batch from pinned host memory, runs the forward, copies logits back."""
+    host_img = torch.from_numpy(images_np).pin_memory().numpy()
+    host_out = torch.empty((B, cfg.classes), dtype=torch.float32).pin_memory().numpy()
+    model.set_mode(args.mode)
+    for _ in range(3):
+        model.forward_host(host_img, host_out)
+    steps = max(5, min(args.steps, 30))
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        model.forward_host(host_img, host_out)
+    dt = time.perf_counter() - t0
+    return {"value": B * steps / dt, "unit": "images/s", "h2d_bytes_per_step": int(host_img.nbytes),
+            "d2h_bytes_per_step": int(host_out.nbytes), "steps": steps,
+            "call": "elasto_forward_host (pinned host buffers, copies + forward + sync per step)"}
+
+
+if __name__ == "__main__":
+    main()

@@ -159,6 +159,27 @@ enum {
 };
 elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value);
 
+/* Per-launch timing (diagnostics). While enabled, forward records a CUDA
+ * event pair around every kernel it launches; elasto_profile_read
+ * synchronises on the last event and returns, for the most recent forward,
+ * one record per launch: what ran, its duration, and its algorithmic work
+ * (multiply-accumulates for contractions, bytes that must cross HBM for the
+ * memory-bound kernels). Events add a few microseconds per forward. */
+enum {
+  ELASTO_K_PATCHIFY = 0, ELASTO_K_GEMM = 1, ELASTO_K_LAYERNORM = 2, ELASTO_K_ATTENTION = 3,
+  ELASTO_K_HEAD = 4, ELASTO_K_IM2COL = 5, ELASTO_K_POOL = 6
+};
+typedef struct {
+  int kind;     /* ELASTO_K_* */
+  int layer;    /* transformer layer / conv block, -1 outside */
+  int m, n, k;  /* GEMM problem (M x N x K); other kernels: rows, cols, 0 */
+  float ms;     /* device duration */
+  double macs;  /* algorithmic multiply-accumulates */
+  double bytes; /* algorithmic HBM bytes (inputs read once + outputs written) */
+} elasto_launch_record;
+elasto_status elasto_profile_enable(elasto_t h, int enable);
+elasto_status elasto_profile_read(elasto_t h, elasto_launch_record* out, int capacity, int* count);
+
 /* Test hook: copy one packed buffer of (mode, layer) to host_dst (bytes must
  * equal its size). ViT `which`: 0 qkv_w bf16 [3w,d], 1 qkv_b fp32 [3w],
  * 2 proj_w bf16 [d,w], 3 fc1_w bf16 [f,d], 4 fc1_b fp32 [f], 5 fc2_w bf16 [d,f]

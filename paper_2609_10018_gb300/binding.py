@@ -44,6 +44,16 @@ class ModeTables(ctypes.Structure):
                 ("conv_kept_a", P_i32), ("n_conv_a", P_i32), ("conv_kept_b", P_i32), ("n_conv_b", P_i32)]
 
 
+K_PATCHIFY, K_GEMM, K_LAYERNORM, K_ATTENTION, K_HEAD, K_IM2COL, K_POOL = range(7)
+KIND_NAMES = {K_PATCHIFY: "patchify", K_GEMM: "gemm", K_LAYERNORM: "layernorm", K_ATTENTION: "attention",
+              K_HEAD: "head", K_IM2COL: "im2col", K_POOL: "pool"}
+
+
+class LaunchRecord(ctypes.Structure):
+    _fields_ = [("kind", c_int), ("layer", c_int), ("m", c_int), ("n", c_int), ("k", c_int),
+                ("ms", ctypes.c_float), ("macs", ctypes.c_double), ("bytes", ctypes.c_double)]
+
+
 class ElastoError(RuntimeError):
     def __init__(self, status: int, where: str, msg: str):
         super().__init__(f"{where} failed with status {status}: {msg}")
@@ -72,6 +82,8 @@ def lib() -> ctypes.CDLL:
         "elasto_destroy": [c_void_p],
         "elasto_query": [c_void_p, c_int, c_int, ctypes.POINTER(c_int64)],
         "elasto_debug_export_packed": [c_void_p, c_int, c_int, c_int, c_void_p, c_size_t],
+        "elasto_profile_enable": [c_void_p, c_int],
+        "elasto_profile_read": [c_void_p, ctypes.POINTER(LaunchRecord), c_int, ctypes.POINTER(c_int)],
         "elasto_op_gemm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
                            c_void_p],
         "elasto_op_layernorm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int],
@@ -216,6 +228,19 @@ def elasto_debug_export_packed(h: int, mode: int, layer: int, which: int, out: n
     return out
 
 
+def elasto_profile_enable(h: int, enable: bool) -> None:
+    _check(lib().elasto_profile_enable(h, 1 if enable else 0), "elasto_profile_enable")
+
+
+def elasto_profile_read(h: int, capacity: int = 1024) -> List[dict]:
+    """Per-launch records of the most recent forward (synchronises)."""
+    buf = (LaunchRecord * capacity)()
+    n = c_int()
+    _check(lib().elasto_profile_read(h, buf, capacity, ctypes.byref(n)), "elasto_profile_read")
+    return [{"kind": KIND_NAMES.get(r.kind, str(r.kind)), "layer": r.layer, "m": r.m, "n": r.n, "k": r.k,
+             "ms": r.ms, "macs": r.macs, "bytes": r.bytes} for r in buf[:n.value]]
+
+
 def elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status=0) -> None:
     _check(lib().elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status), "elasto_op_gemm")
 
@@ -279,6 +304,12 @@ class ElasticModel:
 
     def query(self, what: int, mode: int = 0) -> int:
         return elasto_query(self.handle, what, mode)
+
+    def profile(self, enable: bool) -> None:
+        elasto_profile_enable(self.handle, enable)
+
+    def profile_read(self) -> List[dict]:
+        return elasto_profile_read(self.handle)
 
     def export_packed(self, mode: int, layer: int, which: int, out: np.ndarray) -> np.ndarray:
         return elasto_debug_export_packed(self.handle, mode, layer, which, out)

@@ -84,6 +84,53 @@ elasto_status check_device() {
   return ELASTO_OK;
 }
 
+// ---------------------------------------------------------------- profiler
+cudaError_t Profiler::enable(bool e) {
+  if (e && !ev[0]) {
+    for (int i = 0; i < 2 * kSlots; ++i) {
+      cudaError_t r = cudaEventCreate(&ev[i]);
+      if (r != cudaSuccess) return r;
+    }
+  }
+  on = e;
+  count = 0;
+  return cudaSuccess;
+}
+cudaError_t Profiler::before(cudaStream_t s) {
+  if (!on) return cudaSuccess;
+  if (count >= kSlots) {
+    overflow = true;
+    return cudaSuccess;
+  }
+  return cudaEventRecord(ev[2 * count], s);
+}
+cudaError_t Profiler::after(cudaStream_t s, const elasto_launch_record& r) {
+  if (!on || count >= kSlots) return cudaSuccess;
+  rec[count] = r;
+  cudaError_t e = cudaEventRecord(ev[2 * count + 1], s);
+  ++count;
+  return e;
+}
+elasto_status Profiler::read(elasto_launch_record* out, int capacity, int* n) {
+  if (!on) {
+    set_error("elasto_profile_read: profiling is not enabled");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (count > 0) ELASTO_CUDA_TRY(cudaEventSynchronize(ev[2 * count - 1]));
+  const int m = count < capacity ? count : capacity;
+  for (int i = 0; i < m; ++i) {
+    out[i] = rec[i];
+    ELASTO_CUDA_TRY(cudaEventElapsedTime(&out[i].ms, ev[2 * i], ev[2 * i + 1]));
+  }
+  *n = m;
+  return ELASTO_OK;
+}
+void Profiler::release() {
+  for (int i = 0; i < 2 * kSlots; ++i)
+    if (ev[i]) cudaEventDestroy(ev[i]);
+  on = false;
+}
+
 }  // namespace elasto
 
 using namespace elasto;
@@ -138,6 +185,7 @@ struct elasto_s {
   std::atomic<int> cur{0};
   // CNN state lives behind this pointer (null for ViT)
   CnnModel* cnn = nullptr;
+  Profiler prof;
 };
 
 namespace {
@@ -492,26 +540,64 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   return ELASTO_OK;
 }
 
+elasto_launch_record make_rec(int kind, int layer, int m, int n, int k, double macs, double bytes) {
+  elasto_launch_record r{};
+  r.kind = kind;
+  r.layer = layer;
+  r.m = m;
+  r.n = n;
+  r.k = k;
+  r.macs = macs;
+  r.bytes = bytes;
+  return r;
+}
+
+// GEMM record: A [M,K] and W [N,K] bf16 read once, out [M,N] written (and
+// read too for a residual epilogue).
+elasto_launch_record gemm_rec(int layer, int M, int N, int K, int out_bytes, bool resid) {
+  const double mn = double(M) * N;
+  return make_rec(ELASTO_K_GEMM, layer, M, N, K, mn * K,
+                  2.0 * M * K + 2.0 * N * K + mn * out_bytes * (resid ? 2 : 1));
+}
+
+#define ELASTO_LAUNCH(rec, expr)                 \
+  do {                                           \
+    ELASTO_CUDA_TRY(h->prof.before(s));          \
+    ELASTO_CUDA_TRY(expr);                       \
+    ELASTO_CUDA_TRY(h->prof.after(s, (rec)));    \
+  } while (0)
+
 elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int batch, float* logits) {
   const elasto_model_desc& d = h->d;
   const VitMode& vm = h->modes[h->cur.load(std::memory_order_acquire)];
-  const int n = h->n, D = d.dim, M = batch * n;
-  ELASTO_CUDA_TRY(
-      patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, h->X, h->cls, h->pos, D, s));
-  ELASTO_CUDA_TRY(gemm_launch(h->patch, batch * h->np, s));
+  const int n = h->n, D = d.dim, M = batch * n, Mp = batch * h->np, C = d.classes;
+  const double img_elt = d.weight_dtype == ELASTO_BF16 ? 2 : 4;
+  h->prof.begin();
+  ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, Mp, h->kpe, 0, 0,
+                         double(Mp) * h->kpe * (img_elt + 2) + double(batch) * D * 4),
+                patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, h->X, h->cls,
+                                h->pos, D, s));
+  ELASTO_LAUNCH(gemm_rec(-1, Mp, D, h->kpe, 4, false), gemm_launch(h->patch, Mp, s));
+  const double ln_bytes = double(M) * D * (4 + 2);
   for (int l = 0; l < d.layers; ++l) {
     const VitLayerPack& lp = vm.layers[l];
-    ELASTO_CUDA_TRY(layernorm_launch(h->X, h->ln1_w[l], h->ln1_b[l], h->Y, M, D, s));
+    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, D, 0, 0, ln_bytes),
+                  layernorm_launch(h->X, h->ln1_w[l], h->ln1_b[l], h->Y, M, D, s));
     if (lp.w > 0) {
-      ELASTO_CUDA_TRY(gemm_launch(lp.qkv, M, s));
-      ELASTO_CUDA_TRY(attn_launch(lp.attn, batch, s));
+      ELASTO_LAUNCH(gemm_rec(l, M, 3 * lp.w, D, 2, false), gemm_launch(lp.qkv, M, s));
+      ELASTO_LAUNCH(make_rec(ELASTO_K_ATTENTION, l, M, lp.w, n, 2.0 * batch * n * n * lp.w,
+                             double(M) * lp.w * 2 * 4),
+                    attn_launch(lp.attn, batch, s));
     }
-    ELASTO_CUDA_TRY(gemm_launch(lp.proj, M, s));
-    ELASTO_CUDA_TRY(layernorm_launch(h->X, h->ln2_w[l], h->ln2_b[l], h->Y, M, D, s));
-    if (lp.f > 0) ELASTO_CUDA_TRY(gemm_launch(lp.fc1, M, s));
-    ELASTO_CUDA_TRY(gemm_launch(lp.fc2, M, s));
+    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.w, 4, true), gemm_launch(lp.proj, M, s));
+    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, D, 0, 0, ln_bytes),
+                  layernorm_launch(h->X, h->ln2_w[l], h->ln2_b[l], h->Y, M, D, s));
+    if (lp.f > 0) ELASTO_LAUNCH(gemm_rec(l, M, lp.f_pad, D, 2, false), gemm_launch(lp.fc1, M, s));
+    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.f_pad, 4, true), gemm_launch(lp.fc2, M, s));
   }
-  ELASTO_CUDA_TRY(head_launch(h->X, batch, n, D, h->norm_w, h->norm_b, h->head_w, h->head_b, d.classes, logits, s));
+  ELASTO_LAUNCH(make_rec(ELASTO_K_HEAD, -1, batch, C, D, double(batch) * C * D,
+                         double(batch) * D * 4 + double(C) * D * 4 + double(batch) * C * 4),
+                head_launch(h->X, batch, n, D, h->norm_w, h->norm_b, h->head_w, h->head_b, C, logits, s));
   return ELASTO_OK;
 }
 
@@ -647,6 +733,7 @@ elasto_status elasto_destroy(elasto_t h) {
   cudaDeviceSynchronize();
   if (h->arena) cudaFree(h->arena);
   if (h->cnn) cnn_destroy(h->cnn);
+  h->prof.release();
   delete h;
   return ELASTO_OK;
 }
@@ -676,6 +763,25 @@ elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value) {
     default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
   }
   return ELASTO_OK;
+}
+
+elasto_status elasto_profile_enable(elasto_t h, int enable) {
+  if (!h) {
+    set_error("elasto_profile_enable: null handle");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  Profiler& p = h->cnn ? *cnn_profiler(h->cnn) : h->prof;
+  ELASTO_CUDA_TRY(p.enable(enable != 0));
+  return ELASTO_OK;
+}
+
+elasto_status elasto_profile_read(elasto_t h, elasto_launch_record* out, int capacity, int* count) {
+  if (!h || !out || !count || capacity < 0) {
+    set_error("elasto_profile_read: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  Profiler& p = h->cnn ? *cnn_profiler(h->cnn) : h->prof;
+  return p.read(out, capacity, count);
 }
 
 elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int which, void* host_dst, size_t bytes) {

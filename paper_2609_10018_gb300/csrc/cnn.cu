@@ -6,6 +6,7 @@ namespace elasto {
 
 struct CnnModel {
   int n_modes = 0;
+  Profiler prof;
 };
 
 elasto_status cnn_check_inputs(const elasto_model_desc*, const elasto_weights*, const elasto_mode_tables*, int) {
@@ -23,7 +24,11 @@ int cnn_n_modes(const CnnModel* m) { return m->n_modes; }
 void* cnn_image_stage(CnnModel*) { return nullptr; }
 float* cnn_logit_stage(CnnModel*) { return nullptr; }
 int* cnn_status_word(CnnModel*) { return nullptr; }
-void cnn_destroy(CnnModel* m) { delete m; }
+Profiler* cnn_profiler(CnnModel* m) { return &m->prof; }
+void cnn_destroy(CnnModel* m) {
+  m->prof.release();
+  delete m;
+}
 elasto_status cnn_query(CnnModel*, int, int, int64_t*) { return ELASTO_ERR_UNSUPPORTED; }
 elasto_status cnn_export_packed(CnnModel*, int, int, int, void*, size_t) { return ELASTO_ERR_UNSUPPORTED; }
 

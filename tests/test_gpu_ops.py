@@ -86,7 +86,8 @@ def test_gemm_full_size_outproj_sampled_rows():
     bias = rng.standard_normal(N).astype(np.float32)
     x0 = rng.standard_normal((M, N)).astype(np.float32)
     out = dev(x0)
-    binding.elasto_op_gemm(stream_handle(), dev(A).data_ptr(), dev(W).data_ptr(), dev(bias).data_ptr(),
+    dA, dW, db = dev(A), dev(W), dev(bias)
+    binding.elasto_op_gemm(stream_handle(), dA.data_ptr(), dW.data_ptr(), db.data_ptr(),
                            out.data_ptr(), None, M, N, K, binding.EPI_BIAS_RESID_F32, 0)
     torch.cuda.synchronize()
     rows = np.concatenate([np.arange(0, 130), rng.choice(M, 300, replace=False), np.arange(M - 130, M)])
@@ -103,8 +104,8 @@ def test_layernorm_matches_fp64(rows, d):
     g = (1 + 0.1 * rng.standard_normal(d)).astype(np.float32)
     b = (0.1 * rng.standard_normal(d)).astype(np.float32)
     y = empty_dev((rows, d), torch.uint16)
-    binding.elasto_op_layernorm(stream_handle(), dev(x).data_ptr(), dev(g).data_ptr(), dev(b).data_ptr(),
-                                y.data_ptr(), rows, d)
+    dx, dg, db = dev(x), dev(g), dev(b)
+    binding.elasto_op_layernorm(stream_handle(), dx.data_ptr(), dg.data_ptr(), db.data_ptr(), y.data_ptr(), rows, d)
     torch.cuda.synchronize()
     ref = ov.layer_norm(x.astype(np.float64), g, b)
     got = bf16_to_f64(y)
@@ -117,7 +118,8 @@ def test_softmax_matches_fp64(rows, cols):
     rng = np.random.default_rng(rows * cols)
     x = (rng.standard_normal((rows, cols)) * 4).astype(np.float32)
     y = empty_dev((rows, cols), torch.float32)
-    binding.elasto_op_softmax(stream_handle(), dev(x).data_ptr(), y.data_ptr(), rows, cols)
+    dx = dev(x)
+    binding.elasto_op_softmax(stream_handle(), dx.data_ptr(), y.data_ptr(), rows, cols)
     torch.cuda.synchronize()
     ref = ov.softmax_rows(x.astype(np.float64))
     got = y.cpu().numpy().astype(np.float64)
@@ -135,7 +137,8 @@ def test_attention_matches_fp64(B, n, h):
     qkv = _bf16(rng, (B, n, 3, h, 64))
     out = empty_dev((B, n, h * 64), torch.uint16)
     st = _status()
-    binding.elasto_op_attention(stream_handle(), dev(qkv).data_ptr(), out.data_ptr(), B, n, h, st.data_ptr())
+    dq = dev(qkv)
+    binding.elasto_op_attention(stream_handle(), dq.data_ptr(), out.data_ptr(), B, n, h, st.data_ptr())
     torch.cuda.synchronize()
     assert int(st.item()) == 0
     q = bf16_to_f64(qkv)
@@ -152,7 +155,8 @@ def test_attention_full_size_sampled():
     rng = np.random.default_rng(5)
     qkv = _bf16(rng, (B, n, 3, h, 64))
     out = empty_dev((B, n, h * 64), torch.uint16)
-    binding.elasto_op_attention(stream_handle(), dev(qkv).data_ptr(), out.data_ptr(), B, n, h, 0)
+    dq = dev(qkv)
+    binding.elasto_op_attention(stream_handle(), dq.data_ptr(), out.data_ptr(), B, n, h, 0)
     torch.cuda.synchronize()
     got = bf16_to_f64(out)
     for b in (0, 1, 128, 255):
