@@ -136,6 +136,30 @@ elasto_status elasto_forward(elasto_t h, void* stream, const void* images_device
 elasto_status elasto_forward_host(elasto_t h, void* stream, const void* images_host, int batch,
                                   float* logits_host);
 
+/* The same forward as elasto_forward (ViT handles), for callers that must not
+ * allocate device memory when they run inference: e.g. a process whose
+ * memory manager takes the whole GPU into its own pool at start-up and
+ * forbids later driver allocations, or a latency-critical loop that cannot
+ * absorb the device synchronisation a cudaMalloc/cudaFree may trigger.
+ * The paper has no counterpart; this is a deployment convenience.
+ * It allocates nothing: no cudaMalloc, no cudaFree, no allocating library
+ * routine. All activation scratch lives in one fixed 64 MiB device array
+ * inside the library (present on every GPU that loads it, until exit), so
+ * the handle's own workspace is not used and batch is limited by that array,
+ * not by max_batch: a batch whose scratch does not fit is rejected with
+ * ELASTO_ERR_INVALID_ARG and a message giving the limit for the model and
+ * current mode (e.g. 18 images for the full ViT-B/16 mode, 239 for the tiny ViT).
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) once; make that first call before any stream
+ * capture. Every call uses the same array and it keeps the last call's
+ * contents; each call writes all the scratch it reads, so nothing has to be
+ * cleared, but calls that overlap on the GPU (e.g. on two streams) race on
+ * it: order them on one stream. Asynchronous like elasto_forward; images and
+ * logits are caller-owned device buffers with the same layouts.
+ * Errors: INVALID_ARG, UNSUPPORTED (ResNet-50 handles), CUDA. */
+elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const void* images_device, int batch,
+                                     float* logits_device);
+
 /* Synchronise `stream`, then read and clear the handle's device status word
  * (kernels record ELASTO_ERR_TIMEOUT there instead of hanging). Returns the
  * recorded status or ELASTO_OK. */

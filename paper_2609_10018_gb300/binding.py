@@ -78,6 +78,7 @@ def lib() -> ctypes.CDLL:
         "elasto_get_mode": [c_void_p, ctypes.POINTER(c_int)],
         "elasto_forward": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
         "elasto_forward_host": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
+        "elasto_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
         "elasto_sync_status": [c_void_p, c_void_p],
         "elasto_destroy": [c_void_p],
         "elasto_query": [c_void_p, c_int, c_int, ctypes.POINTER(c_int64)],
@@ -199,6 +200,11 @@ def elasto_get_mode(h: int) -> int:
 
 def elasto_forward(h: int, stream: int, images_ptr: int, batch: int, logits_ptr: int) -> None:
     _check(lib().elasto_forward(h, stream, images_ptr, batch, logits_ptr), "elasto_forward")
+
+
+def elasto_forward_noalloc(h: int, stream: int, images_ptr: int, batch: int, logits_ptr: int) -> None:
+    """Forward with the library's fixed static scratch; allocates nothing."""
+    _check(lib().elasto_forward_noalloc(h, stream, images_ptr, batch, logits_ptr), "elasto_forward_noalloc")
 
 
 def elasto_forward_host(h: int, stream: int, images: np.ndarray, batch: int, logits: np.ndarray) -> None:

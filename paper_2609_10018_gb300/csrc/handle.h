@@ -1,0 +1,58 @@
+// Layout of an elastic-model handle (shared by the C-ABI translation units).
+#pragma once
+#include <atomic>
+#include <vector>
+
+#include "common.h"
+#include "elasto_internal.h"
+
+namespace elasto {
+
+// One layer of one mode: kept widths, packed weights, launch plans.
+struct VitLayerPack {
+  int w = 0;       // kept heads * 64
+  int f = 0;       // kept MLP channels
+  int f_pad = 0;   // f rounded up to a multiple of 8 (zero rows/cols; GELU(0) = 0)
+  bf16* qkv_w = nullptr;
+  float* qkv_b = nullptr;
+  bf16* proj_w = nullptr;
+  bf16* fc1_w = nullptr;
+  float* fc1_b = nullptr;
+  bf16* fc2_w = nullptr;
+  GemmPlan qkv, proj, fc1, fc2;
+  AttnPlan attn;
+};
+
+struct VitMode {
+  std::vector<VitLayerPack> layers;
+  size_t packed_bytes = 0;
+  int64_t macs = 0;
+  int launches = 0;
+};
+
+}  // namespace elasto
+
+struct elasto_s {
+  elasto_model_desc d{};
+  int dev = 0;
+  int n = 0, np = 0, kpe = 0;
+  char* arena = nullptr;
+  size_t arena_bytes = 0, shared_bytes = 0, workspace_bytes = 0;
+  // shared (mode-independent) parameters
+  elasto::bf16* patch_w = nullptr;
+  float *patch_b = nullptr, *cls = nullptr, *pos = nullptr, *norm_w = nullptr, *norm_b = nullptr;
+  float *head_w = nullptr, *head_b = nullptr;
+  std::vector<float*> ln1_w, ln1_b, proj_b, ln2_w, ln2_b, fc2_b;
+  // workspace
+  float* X = nullptr;
+  elasto::bf16 *Y = nullptr, *QKV = nullptr, *O = nullptr, *H = nullptr, *P = nullptr;
+  void* img_stage = nullptr;
+  float* logit_stage = nullptr;
+  int* status = nullptr;
+  elasto::GemmPlan patch;
+  std::vector<elasto::VitMode> modes;
+  std::atomic<int> cur{0};
+  // CNN state lives behind this pointer (null for ViT)
+  elasto::CnnModel* cnn = nullptr;
+  elasto::Profiler prof;
+};
