@@ -46,7 +46,7 @@ def parse_args():
     p.add_argument("--impl", choices=["elasto", "reference"], default="elasto")
     p.add_argument("--batch", type=int, default=256)
     p.add_argument("--mode", type=int, default=0)
-    p.add_argument("--quick", action="store_true", help="headline only: skip per-mode sweep, latency, baseline")
+    p.add_argument("--quick", action="store_true", help="headline only: skip per-mode sweep, latency, e2e, baseline")
     return p.parse_args()
 
 
@@ -344,8 +344,6 @@ def main():
         line["mode_switch_us"] = mode_switch(model, cfg, tables, torch, binding)
         line["e2e"] = e2e(model, cfg, images_np, B, args, torch, binding)
         line["cpu_baseline"] = oracle_cpu_baseline(cfg)
-    elif rank == 0:
-        line["e2e"] = e2e(model, cfg, images_np, B, args, torch, binding)
     model.close()
     if rank == 0:
         print(json.dumps(line))

@@ -32,7 +32,7 @@ int num_sms();  // of the current device
 // 2-D bf16 tensor [outer][inner] (inner contiguous, row stride in bytes),
 // box {box_inner, box_outer}, 128-byte swizzle, out-of-bounds reads as zero.
 bool encode_tmap_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_stride_bytes,
-                    uint32_t box_inner, uint32_t box_outer);
+                    uint32_t box_inner, uint32_t box_outer, bool fp32 = false);
 // 3-D bf16 tensor [d2][d1][d0] with byte strides s1 (between d1 rows) and s2.
 bool encode_tmap_3d(CUtensorMap* tm, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1,
                     uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2);
@@ -60,17 +60,20 @@ struct GemmArgs {
   int tokens;             // PATCH: tokens per image (patches + 1)
   const float* pos;       // PATCH: [tokens, N]
   int* status;
+  int stages;             // operand ring depth (<= 4)
+  int cbufs;              // output staging buffers (16 KB each) for the TMA-store epilogues
 };
 
 struct GemmPlan {
   CUtensorMap tmA, tmB;
+  CUtensorMap tmC;        // output [M_cap, ldo] (bf16 or fp32), box 128 B x 128 rows, 128B swizzle
   GemmArgs args;          // M here is the capacity the A map was encoded for
   int epi = 0;
   bool valid = false;
 };
 
 // Pick the N tile for an M x N problem.
-int gemm_pick_bn(int M, int N);
+int gemm_pick_bn(int M, int N, int step = 32);
 // Build maps/arguments for out = epi(A[M_cap, K] W[N, K]^T). A and W must stay
 // allocated for the plan's life.
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,

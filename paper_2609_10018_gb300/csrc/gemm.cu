@@ -9,15 +9,23 @@
 // Design (sm_103a):
 //  - persistent grid, one CTA per SM, static round-robin over 128 x bn tiles
 //    (N tile index fastest so the CTAs running together share A rows in L2);
-//  - warp 0 lane 0: TMA producer, 4-stage ring of 128x64 (A) and bn x 64 (B)
-//    bf16 tiles with the 128-byte swizzle, one mbarrier pair per stage;
+//  - warp 0 lane 0: TMA producer, ring of 128x64 (A) and bn x 64 (B) bf16
+//    tiles with the 128-byte swizzle, one mbarrier pair per stage;
 //  - warp 1 lane 0: issues tcgen05.mma (M=128, N=bn, K=16) into one of two
 //    TMEM accumulators (2 x 256 fp32 columns), commits stages back to the
 //    producer and finished accumulators to the epilogue;
 //  - warps 2-5: epilogue. Each warp owns one 32-lane quarter of TMEM (= 32
-//    rows of the tile), reads 32 columns at a time, transposes them through a
-//    padded shared-memory tile so that global stores are row-contiguous, and
-//    applies bias / GELU / residual / ReLU / position embedding.
+//    rows of the tile); each thread owns one row.
+//    * bf16 outputs (QKV, FC1+GELU, conv+ReLU) and the fp32 residual stream
+//      (out-proj, FC2): the thread writes its row of a 128-row x 128-byte
+//      chunk into a 128B-swizzled staging buffer in shared memory (bank
+//      conflict free 16-byte stores) and one thread stores the chunk with a
+//      TMA tensor store. For the residual, the old rows of X are brought into
+//      the same staging buffer by TMA loads issued several chunks ahead, so
+//      the read-modify-write of X runs at full memory parallelism.
+//    * the remaining epilogues (fp32 out, patch rows with position
+//      embedding, bf16 residual + ReLU) transpose through padded shared memory
+//      for row-contiguous stores.
 //  Every mbarrier wait is bounded; a timeout records ELASTO_ERR_TIMEOUT.
 #include "common.h"
 #include "ptx.cuh"
@@ -26,32 +34,109 @@ namespace elasto {
 
 namespace {
 
-constexpr int BM = 128, BK = 64, STAGES = 4, MAX_BN = 256, THREADS = 192;
+constexpr int BM = 128, BK = 64, MAX_STAGES = 4, MAX_BN = 256;
+constexpr int EPI_THREADS = 256;                 // 8 epilogue warps, two per TMEM lane quarter
+constexpr int THREADS = 64 + EPI_THREADS;
 constexpr int A_STAGE = BM * BK * 2;        // 16 KB
 constexpr int B_STAGE = MAX_BN * BK * 2;    // 32 KB
+constexpr int CBUF = BM * 128;              // 16 KB staging chunk (128 rows x 128 B)
+constexpr int POOL = 224 * 1024;            // operand ring + staging buffers
+constexpr int MAX_CBUFS = 8;
 constexpr int EPI_LD = 33;                  // padded row of the transpose tile
 constexpr int EPI_TILE = 32 * EPI_LD;       // floats per epilogue warp
 constexpr int TMEM_COLS = 512;
-constexpr size_t SMEM_BYTES = 1024 + STAGES * (A_STAGE + B_STAGE) + 4 * EPI_TILE * 4 + 256;
+constexpr size_t SMEM_BYTES = 1024 + POOL + 512;
 
-__device__ __forceinline__ float gelu_erf(float x) { return 0.5f * x * (1.0f + erff(x * 0.70710678118654752f)); }
+// Exact (erf) GELU, phi in Eq. 5. erf by Abramowitz & Stegun, Handbook of
+// Mathematical Functions, formula 7.1.26: for z >= 0,
+//   erf(z) = 1 - (a1 t + a2 t^2 + a3 t^3 + a4 t^4 + a5 t^5) exp(-z^2), t = 1 / (1 + p z),
+// with |error| <= 1.5e-7 (far below the bf16 rounding of the output), and
+// erf(-z) = -erf(z).
+__device__ __forceinline__ float gelu_erf(float x) {
+  const float z = fabsf(x) * 0.70710678118654752f;
+  const float t = __fdividef(1.0f, fmaf(0.3275911f, z, 1.0f));
+  const float poly =
+      t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, 1.061405429f, -1.453152027f), 1.421413741f), -0.284496736f), 0.254829592f);
+  const float e = exp2f(-z * z * 1.4426950408889634f);
+  const float erf_abs = fmaf(-poly, e, 1.0f);
+  const float half_x = 0.5f * x;
+  return fmaf(half_x, copysignf(erf_abs, x), half_x);
+}
+
+template <int EPI>
+struct EpiTraits {
+  static constexpr bool tma = EPI == EPI_BIAS_BF16 || EPI == EPI_BIAS_GELU_BF16 || EPI == EPI_BIAS_RELU_BF16 ||
+                              EPI == EPI_BIAS_RESID_F32;
+  static constexpr bool f32 = EPI == EPI_BIAS_RESID_F32;
+  static constexpr bool resid = EPI == EPI_BIAS_RESID_F32;
+  static constexpr int cw = f32 ? 32 : 64;  // columns per 128-byte staging chunk
+};
+
+template <int EPI>
+__device__ __forceinline__ float epi_act(float v) {
+  if constexpr (EPI == EPI_BIAS_GELU_BF16) return gelu_erf(v);
+  if constexpr (EPI == EPI_BIAS_RELU_BF16) return fmaxf(v, 0.0f);
+  return v;
+}
+
+// W consecutive bias values starting at column col (zero past N or if null).
+template <int W>
+__device__ __forceinline__ void load_bias(const float* bias, int col, int N, float (&b)[W]) {
+  if (bias && col + W <= N) {
+    const float4* p = reinterpret_cast<const float4*>(bias + col);
+#pragma unroll
+    for (int j = 0; j < W / 4; ++j) {
+      const float4 v = __ldg(p + j);
+      b[4 * j] = v.x;
+      b[4 * j + 1] = v.y;
+      b[4 * j + 2] = v.z;
+      b[4 * j + 3] = v.w;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < W; ++j) b[j] = (bias && col + j < N) ? __ldg(bias + col + j) : 0.0f;
+  }
+}
+
+// Walks this CTA's sequence of (tile, chunk) pairs, skipping chunks past N.
+struct ChunkIter {
+  int t, c;
+  bool valid;
+  __device__ __forceinline__ void init(int tiles) {
+    t = blockIdx.x;
+    c = 0;
+    valid = t < tiles;
+  }
+  __device__ __forceinline__ void advance(int tiles, int nt, int bn, int cw, int N) {
+    const int n0 = (t % nt) * bn;
+    ++c;
+    if (c * cw >= bn || n0 + c * cw >= N) {
+      c = 0;
+      t += gridDim.x;
+      valid = t < tiles;
+    }
+  }
+};
 
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const GemmArgs args) {
+                   const __grid_constant__ CUtensorMap tmC, const GemmArgs args) {
+  using TR = EpiTraits<EPI>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int S = args.stages, E = args.cbufs;
   uint8_t* sA = smem;
-  uint8_t* sB = smem + STAGES * A_STAGE;
-  float* sEpi = reinterpret_cast<float*>(sB + STAGES * B_STAGE);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(sEpi + 4 * EPI_TILE);
+  uint8_t* sB = smem + S * A_STAGE;
+  uint8_t* sC = sB + S * B_STAGE;  // E staging chunks, or the transpose tiles
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + POOL);
   uint64_t* full = bars;
-  uint64_t* empty = bars + STAGES;
-  uint64_t* tfull = bars + 2 * STAGES;
+  uint64_t* empty = bars + MAX_STAGES;
+  uint64_t* tfull = bars + 2 * MAX_STAGES;
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* rfull = drain + 1;  // MAX_CBUFS residual-landed barriers
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rfull + MAX_CBUFS);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int M = args.M, N = args.N, bn = args.bn;
@@ -60,24 +145,28 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int tiles = mt * nt;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < MAX_STAGES; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], 4);
+      mbar_init(&tempty[a], TR::tma ? 8 : 4);
     }
     mbar_init(drain, 1);
+    for (int e = 0; e < MAX_CBUFS; ++e) mbar_init(&rfull[e], 1);
     fence_barrier_init();
   }
   if (warp == 0) {
     tmem_alloc(tmem_slot, TMEM_COLS);
     tmem_relinquish();
   }
-  if (warp == 1 && lane == 0 && nk > 0) {
-    tma_prefetch_desc(&tmA);
-    tma_prefetch_desc(&tmB);
+  if (warp == 1 && lane == 0) {
+    if (nk > 0) {
+      tma_prefetch_desc(&tmA);
+      tma_prefetch_desc(&tmB);
+    }
+    if constexpr (TR::tma) tma_prefetch_desc(&tmC);
   }
   tc_fence_before();
   __syncthreads();
@@ -103,18 +192,18 @@ __global__ void __launch_bounds__(THREADS, 1)
           tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
           tma_load_2d(sB + stage * B_STAGE, &tmB, &full[stage], kb * BK, n0);
           ++issued;
-          if (++stage == STAGES) {
+          if (++stage == S) {
             stage = 0;
             phase ^= 1;
           }
         }
       }
       if (!ok) record_status(args.status, ELASTO_ERR_TIMEOUT);
-      // Drain: make sure no copy is still landing in shared memory when the
-      // CTA exits (returns at once on the normal path).
-      for (int i = 0; i < STAGES && i < issued; ++i) {
+      // Drain: no copy may still be landing in shared memory when the CTA
+      // exits (returns at once on the normal path).
+      for (int i = 0; i < S && i < issued; ++i) {
         if (stage == 0) {
-          stage = STAGES;
+          stage = S;
           phase ^= 1;
         }
         --stage;
@@ -156,7 +245,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           issued = true;
           tc_commit(&empty[stage]);
-          if (++stage == STAGES) {
+          if (++stage == S) {
             stage = 0;
             phase ^= 1;
           }
@@ -170,10 +259,154 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_wait(drain, 0);
       }
     }
+  } else if constexpr (TR::tma) {
+    // ------------------------------------------------------------ TMA-store epilogue
+    constexpr int CW = TR::cw;
+    constexpr int HW = CW / 2;              // columns of a chunk handled by one warp group
+    const int q = warp & 3;                 // TMEM lane quarter
+    const int g = (warp - 2) >> 2;          // warp group: first or second half of each chunk
+    const int r = q * 32 + lane;            // row within the tile
+    const bool elected = threadIdx.x == 64;
+    const int cpt = bn / CW;
+    const uint32_t row_tm = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
+    // One thread takes every wait decision and shares it through `verdict`,
+    // so the 128 epilogue threads always agree on whether to continue and
+    // the named barriers below can never be left one arrival short.
+    volatile int* verdict = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    ChunkIter pf;  // residual prefetch iterator (elected thread only)
+    pf.init(tiles);
+    long loads = 0, consumed = 0;
+    if constexpr (TR::resid) {
+      if (elected) {
+        for (int e = 0; e < E && pf.valid; ++e) {
+          mbar_expect_tx(&rfull[e], CBUF);
+          tma_load_2d(sC + e * CBUF, &tmC, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
+          pf.advance(tiles, nt, bn, CW, N);
+          ++loads;
+        }
+      }
+    }
+    int e = 0;
+    uint32_t rph = 0;
+    bool ok = true;
+    int local = 0;
+    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++local) {
+      const int acc = local & 1;
+      const uint32_t use = static_cast<uint32_t>(local >> 1);
+      if (elected) *verdict = mbar_wait(&tfull[acc], use & 1) ? 1 : 0;
+      named_bar_sync(1, EPI_THREADS);
+      if (!*verdict) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const int m0 = (t / nt) * BM, n0 = (t % nt) * bn;
+      const uint32_t acc_tm = row_tm + acc * MAX_BN;
+      int nvalid = 0;
+      while (nvalid < cpt && n0 + nvalid * CW < N) ++nvalid;
+      for (int c = 0; c < nvalid; ++c) {
+        uint8_t* buf = sC + e * CBUF;
+        uint8_t* rowp = buf + r * 128;
+        if constexpr (TR::resid) {
+          if (elected) *verdict = mbar_wait(&rfull[e], rph) ? 1 : 0;
+          named_bar_sync(1, EPI_THREADS);
+          if (!*verdict) {
+            ok = false;
+            break;
+          }
+          ++consumed;
+        }
+        {
+          // this thread: row r, columns [g*HW, g*HW + HW) of the chunk = 16-byte
+          // chunks 4g .. 4g+3 of the 128-byte staging row
+          uint32_t v[HW];
+          if (nk > 0) {
+            if constexpr (HW == 32)
+              tmem_ld_32x32b_x32(acc_tm + c * CW + g * HW, v);
+            else
+              tmem_ld_16(acc_tm + c * CW + g * HW, v);
+            tmem_ld_wait();
+          } else {
+#pragma unroll
+            for (int j = 0; j < HW; ++j) v[j] = 0u;
+          }
+          if (c == nvalid - 1) {  // last TMEM read of this tile
+            tc_fence_before();
+            if (lane == 0) mbar_arrive(&tempty[acc]);
+          }
+          float bb[HW];
+          load_bias<HW>(args.bias, n0 + c * CW + g * HW, N, bb);
+          if constexpr (TR::f32) {
+            // 16 fp32; X_old arrived by TMA into the same swizzled row
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              float4* p = reinterpret_cast<float4*>(rowp + (((4 * g + j) ^ (r & 7)) << 4));
+              float4 o = *p;
+              o.x += __uint_as_float(v[4 * j]) + bb[4 * j];
+              o.y += __uint_as_float(v[4 * j + 1]) + bb[4 * j + 1];
+              o.z += __uint_as_float(v[4 * j + 2]) + bb[4 * j + 2];
+              o.w += __uint_as_float(v[4 * j + 3]) + bb[4 * j + 3];
+              *p = o;
+            }
+          } else {
+            // 32 bf16
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              uint4 pk;
+              pk.x = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 0]) + bb[8 * j + 0]),
+                                 epi_act<EPI>(__uint_as_float(v[8 * j + 1]) + bb[8 * j + 1]));
+              pk.y = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 2]) + bb[8 * j + 2]),
+                                 epi_act<EPI>(__uint_as_float(v[8 * j + 3]) + bb[8 * j + 3]));
+              pk.z = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 4]) + bb[8 * j + 4]),
+                                 epi_act<EPI>(__uint_as_float(v[8 * j + 5]) + bb[8 * j + 5]));
+              pk.w = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 6]) + bb[8 * j + 6]),
+                                 epi_act<EPI>(__uint_as_float(v[8 * j + 7]) + bb[8 * j + 7]));
+              *reinterpret_cast<uint4*>(rowp + (((4 * g + j) ^ (r & 7)) << 4)) = pk;
+            }
+          }
+        }
+        fence_async_smem();
+        named_bar_sync(1, EPI_THREADS);
+        if (elected) {
+          tma_store_2d(&tmC, buf, n0 + c * CW, m0);
+          bulk_commit();
+          bulk_wait_read_all();  // buffer e may be refilled
+          if constexpr (TR::resid) {
+            if (pf.valid) {
+              mbar_expect_tx(&rfull[e], CBUF);
+              tma_load_2d(buf, &tmC, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
+              pf.advance(tiles, nt, bn, CW, N);
+              ++loads;
+            }
+          }
+        }
+        if (++e == E) {
+          e = 0;
+          rph ^= 1;
+        }
+      }
+    }
+    if (!ok && elected) record_status(args.status, ELASTO_ERR_TIMEOUT);
+    if (elected) {
+      bulk_wait_all();
+      if constexpr (TR::resid) {
+        // Residual loads issued for chunks never consumed (only on the abort
+        // path): let them land before the CTA releases its shared memory.
+        for (long i = consumed; i < loads; ++i) {
+          mbar_wait(&rfull[e], rph);
+          if (++e == E) {
+            e = 0;
+            rph ^= 1;
+          }
+        }
+      }
+    }
   } else {
-    // ------------------------------------------------------------ epilogue
+    // ------------------------------------------------------------ transpose epilogue
+    // (warps 2-5 only; warps 6-9 have nothing to do here)
+    if (warp < 6) {
     const int q = warp & 3;  // TMEM lane quarter this warp may access
-    float* st = sEpi + (warp - 2) * EPI_TILE;
+    float* st = reinterpret_cast<float*>(sC) + (warp - 2) * EPI_TILE;
     int local = 0;
     for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++local) {
       const int acc = local & 1;
@@ -198,24 +431,12 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) st[lane * EPI_LD + j] = __uint_as_float(r[j]);
         __syncwarp();
-        if constexpr (EPI == EPI_BIAS_RESID_F32 || EPI == EPI_BIAS_F32 || EPI == EPI_PATCH_POS_F32) {
+        if constexpr (EPI == EPI_BIAS_F32 || EPI == EPI_PATCH_POS_F32) {
           const int col = n0 + c + lane;
           const bool cok = col < N;
           const float bv = (cok && args.bias) ? args.bias[col] : 0.0f;
           float* out = static_cast<float*>(args.out);
-          if constexpr (EPI == EPI_BIAS_RESID_F32) {
-            float old[32];
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int row = row0 + i;
-              old[i] = (cok && row < M) ? out[static_cast<size_t>(row) * args.ldo + col] : 0.0f;
-            }
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int row = row0 + i;
-              if (cok && row < M) out[static_cast<size_t>(row) * args.ldo + col] = old[i] + (st[i * EPI_LD + lane] + bv);
-            }
-          } else if constexpr (EPI == EPI_BIAS_F32) {
+          if constexpr (EPI == EPI_BIAS_F32) {
 #pragma unroll 8
             for (int i = 0; i < 32; ++i) {
               const int row = row0 + i;
@@ -234,6 +455,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
           }
         } else {
+          // EPI_BIAS_RESID_RELU_BF16
           const int cp = (lane & 15) * 2;
           const int col = n0 + c + cp;
           const bool cok = col < N;
@@ -245,20 +467,10 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int rr = 2 * i + (lane >> 4);
             const int row = row0 + rr;
             if (!(cok && row < M)) continue;
-            float v0 = st[rr * EPI_LD + cp] + b0;
-            float v1 = st[rr * EPI_LD + cp + 1] + b1;
-            if constexpr (EPI == EPI_BIAS_GELU_BF16) {
-              v0 = gelu_erf(v0);
-              v1 = gelu_erf(v1);
-            } else if constexpr (EPI == EPI_BIAS_RELU_BF16) {
-              v0 = fmaxf(v0, 0.0f);
-              v1 = fmaxf(v1, 0.0f);
-            } else if constexpr (EPI == EPI_BIAS_RESID_RELU_BF16) {
-              const __nv_bfloat162 rv =
-                  *reinterpret_cast<const __nv_bfloat162*>(args.resid + static_cast<size_t>(row) * args.ldr + col);
-              v0 = fmaxf(v0 + __bfloat162float(rv.x), 0.0f);
-              v1 = fmaxf(v1 + __bfloat162float(rv.y), 0.0f);
-            }
+            const __nv_bfloat162 rv =
+                *reinterpret_cast<const __nv_bfloat162*>(args.resid + static_cast<size_t>(row) * args.ldr + col);
+            const float v0 = fmaxf(st[rr * EPI_LD + cp] + b0 + __bfloat162float(rv.x), 0.0f);
+            const float v1 = fmaxf(st[rr * EPI_LD + cp + 1] + b1 + __bfloat162float(rv.y), 0.0f);
             out[(static_cast<size_t>(row) * args.ldo + col) >> 1] = pack_bf16x2(v0, v1);
           }
         }
@@ -266,6 +478,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       tc_fence_before();
       if (lane == 0) mbar_arrive(&tempty[acc]);
+    }
     }
   }
   __syncthreads();
@@ -282,7 +495,7 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   a.M = M;
   const int tiles = ((M + BM - 1) / BM) * ((a.N + a.bn - 1) / a.bn);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, a);
+  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmC, a);
   return cudaGetLastError();
 }
 
@@ -305,13 +518,13 @@ cudaError_t gemm_init_attributes() {
   return cudaSuccess;
 }
 
-int gemm_pick_bn(int M, int N) {
+int gemm_pick_bn(int M, int N, int step) {
   // Estimated time ~ waves x (bn + fixed per-tile overhead); ties prefer wider tiles.
   const int sms = num_sms() > 0 ? num_sms() : 148;
   const int mt = (M + BM - 1) / BM;
   int best = 256;
   long best_cost = -1;
-  for (int bn = 256; bn >= 32; bn -= 32) {
+  for (int bn = 256; bn >= step; bn -= step) {
     const long tiles = static_cast<long>(mt) * ((N + bn - 1) / bn);
     const long waves = (tiles + sms - 1) / sms;
     const long cost = waves * (bn + 32);
@@ -334,16 +547,36 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     return ELASTO_ERR_UNSUPPORTED;
   }
   *p = GemmPlan{};
+  const bool tma_out = epi == EPI_BIAS_BF16 || epi == EPI_BIAS_GELU_BF16 || epi == EPI_BIAS_RELU_BF16 ||
+                       epi == EPI_BIAS_RESID_F32;
+  const bool f32_out = epi == EPI_BIAS_RESID_F32;
   GemmArgs& a = p->args;
   a.M = M_cap;
   a.N = N;
   a.K = K;
-  a.bn = gemm_pick_bn(M_cap, N);
+  // bf16 staging chunks are 64 columns wide: their tiles are multiples of 64
+  a.bn = gemm_pick_bn(M_cap, N, (tma_out && !f32_out) ? 64 : 32);
   a.bias = bias;
   a.out = out;
   a.ldo = ldo;
   a.status = status;
   p->epi = epi;
+  if (tma_out) {
+    // residual GEMMs: 3 operand stages and 5 staging chunks fetched ahead;
+    // the others: 4 stages and 2 staging chunks.
+    a.stages = f32_out ? 3 : 4;
+    a.cbufs = (POOL - a.stages * (A_STAGE + B_STAGE)) / CBUF;
+    if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
+    if (ldo % 8 != 0 ||
+        !encode_tmap_2d(&p->tmC, out, ldo, M_cap, static_cast<uint64_t>(ldo) * (f32_out ? 4 : 2),
+                        f32_out ? 32 : 64, BM, f32_out)) {
+      set_error("gemm_plan: output tensor map (alignment or size)");
+      return ELASTO_ERR_UNSUPPORTED;
+    }
+  } else {
+    a.stages = MAX_STAGES;
+    a.cbufs = 0;
+  }
   if (K > 0) {
     if (!encode_tmap_2d(&p->tmA, A, K, M_cap, static_cast<uint64_t>(K) * 2, BK, BM) ||
         !encode_tmap_2d(&p->tmB, W, K, N, static_cast<uint64_t>(K) * 2, BK, a.bn)) {
