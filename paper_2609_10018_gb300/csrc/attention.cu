@@ -164,6 +164,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t lane_base = tmem + (static_cast<uint32_t>(qq * 32) << 16) + t * 256;
       const float kscale = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
       const int n_read = (n + 31) & ~31;                  // columns read (<= 256)
+      const int n_full = n & ~31;                         // columns in whole valid chunks
       int i = 0;
       for (int item = blockIdx.x; item < items; item += gridDim.x, ++i) {
         const uint32_t ph = i & 1;
@@ -173,36 +174,58 @@ __global__ void __launch_bounds__(THREADS, 1)
           break;
         }
         tc_fence_after();
-        // pass 1: row max over the valid keys
-        float mx = -INFINITY;
-        for (int c = 0; c < n_read; c += 64) {
+        // pass 1: row max over the valid keys (unmasked over whole 32-column
+        // chunks, four independent partial maxima)
+        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+        int c = 0;
+        for (; c + 64 <= n_full; c += 64) {
           uint32_t v[32], u[32];
           tmem_ld_32x32b_x32(lane_base + c, v);
-          if (c + 32 < n_read) tmem_ld_32x32b_x32(lane_base + c + 32, u);
+          tmem_ld_32x32b_x32(lane_base + c + 32, u);
           tmem_ld_wait();
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
-            if (c + j < n) mx = fmaxf(mx, __uint_as_float(v[j]));
-            if (c + 32 + j < n) mx = fmaxf(mx, __uint_as_float(u[j]));
+            m4[j & 3] = fmaxf(m4[j & 3], __uint_as_float(v[j]));
+            m4[j & 3] = fmaxf(m4[j & 3], __uint_as_float(u[j]));
           }
         }
-        // pass 2: numerators and row sum; P as bf16 pairs into TMEM columns
-        // [c/2, c/2 + 16), all of which pass 2 has already read
-        const float mxs = mx * kscale;
-        float sum = 0.0f;
-        for (int c = 0; c < n_read; c += 32) {
-          uint32_t v[32], pk[16];
+        for (; c < n_read; c += 32) {
+          uint32_t v[32];
           tmem_ld_32x32b_x32(lane_base + c, v);
           tmem_ld_wait();
 #pragma unroll
-          for (int j = 0; j < 32; j += 2) {
-            const float p0 = (c + j < n) ? exp2f(fmaf(__uint_as_float(v[j]), kscale, -mxs)) : 0.0f;
-            const float p1 = (c + j + 1 < n) ? exp2f(fmaf(__uint_as_float(v[j + 1]), kscale, -mxs)) : 0.0f;
-            sum += p0 + p1;
-            pk[j >> 1] = pack_bf16x2(p0, p1);
+          for (int j = 0; j < 32; ++j)
+            if (c + j < n) m4[j & 3] = fmaxf(m4[j & 3], __uint_as_float(v[j]));
+        }
+        const float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+        // pass 2: numerators and row sum; P as bf16 pairs into TMEM columns
+        // [c/2, c/2 + 16), all of which pass 2 has already read
+        const float mxs = mx * kscale;
+        float s4[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        for (c = 0; c < n_read; c += 32) {
+          uint32_t v[32], pk[16];
+          tmem_ld_32x32b_x32(lane_base + c, v);
+          tmem_ld_wait();
+          if (c + 32 <= n) {
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) {
+              const float p0 = ex2_approx(fmaf(__uint_as_float(v[j]), kscale, -mxs));
+              const float p1 = ex2_approx(fmaf(__uint_as_float(v[j + 1]), kscale, -mxs));
+              s4[(j >> 1) & 3] += p0 + p1;
+              pk[j >> 1] = pack_bf16x2(p0, p1);
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 32; j += 2) {
+              const float p0 = (c + j < n) ? ex2_approx(fmaf(__uint_as_float(v[j]), kscale, -mxs)) : 0.0f;
+              const float p1 = (c + j + 1 < n) ? ex2_approx(fmaf(__uint_as_float(v[j + 1]), kscale, -mxs)) : 0.0f;
+              s4[(j >> 1) & 3] += p0 + p1;
+              pk[j >> 1] = pack_bf16x2(p0, p1);
+            }
           }
           tmem_st_16(lane_base + (c >> 1), pk);
         }
+        const float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
         tmem_st_wait();
         tc_fence_before();
         mbar_arrive(&p_full[t]);

@@ -35,7 +35,7 @@ namespace elasto {
 namespace {
 
 constexpr int BM = 128, BK = 64, MAX_STAGES = 4, MAX_BN = 256;
-constexpr int EPI_THREADS = 256;                 // 8 epilogue warps, two per TMEM lane quarter
+constexpr int EPI_THREADS = 512;                 // 16 epilogue warps, four per TMEM lane quarter
 constexpr int THREADS = 64 + EPI_THREADS;
 constexpr int A_STAGE = BM * BK * 2;        // 16 KB
 constexpr int B_STAGE = MAX_BN * BK * 2;    // 32 KB
@@ -51,13 +51,16 @@ constexpr size_t SMEM_BYTES = 1024 + POOL + 512;
 // Mathematical Functions, formula 7.1.26: for z >= 0,
 //   erf(z) = 1 - (a1 t + a2 t^2 + a3 t^3 + a4 t^4 + a5 t^5) exp(-z^2), t = 1 / (1 + p z),
 // with |error| <= 1.5e-7 (far below the bf16 rounding of the output), and
-// erf(-z) = -erf(z).
+// erf(-z) = -erf(z). Here z = |x| / sqrt(2); with u = z * sqrt(log2 e) the
+// exponential is 2^(-u^2) and p z = (p / sqrt(log2 e)) u.
 __device__ __forceinline__ float gelu_erf(float x) {
-  const float z = fabsf(x) * 0.70710678118654752f;
-  const float t = __fdividef(1.0f, fmaf(0.3275911f, z, 1.0f));
+  constexpr float kU = 0.70710678118654752f * 1.2011224087864498f;  // 1/sqrt(2) * sqrt(log2 e)
+  constexpr float kP = 0.3275911f / 1.2011224087864498f;
+  const float u = fabsf(x) * kU;
+  const float t = __fdividef(1.0f, fmaf(kP, u, 1.0f));
   const float poly =
       t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, 1.061405429f, -1.453152027f), 1.421413741f), -0.284496736f), 0.254829592f);
-  const float e = exp2f(-z * z * 1.4426950408889634f);
+  const float e = ex2_approx(-u * u);
   const float erf_abs = fmaf(-poly, e, 1.0f);
   const float half_x = 0.5f * x;
   return fmaf(half_x, copysignf(erf_abs, x), half_x);
@@ -151,7 +154,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], TR::tma ? 8 : 4);
+      mbar_init(&tempty[a], TR::tma ? EPI_THREADS / 32 : 4);
     }
     mbar_init(drain, 1);
     for (int e = 0; e < MAX_CBUFS; ++e) mbar_init(&rfull[e], 1);
@@ -262,9 +265,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else if constexpr (TR::tma) {
     // ------------------------------------------------------------ TMA-store epilogue
     constexpr int CW = TR::cw;
-    constexpr int HW = CW / 2;              // columns of a chunk handled by one warp group
+    constexpr int NG = EPI_THREADS / 128;   // warp groups sharing each chunk
+    constexpr int HW = CW / NG;             // columns of a chunk handled by one thread
+    constexpr int NC = HW * (TR::f32 ? 4 : 2) / 16;  // 16-byte pieces per thread
     const int q = warp & 3;                 // TMEM lane quarter
-    const int g = (warp - 2) >> 2;          // warp group: first or second half of each chunk
+    const int g = (warp - 2) >> 2;          // warp group: which part of each chunk
     const int r = q * 32 + lane;            // row within the tile
     const bool elected = threadIdx.x == 64;
     const int cpt = bn / CW;
@@ -275,7 +280,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     volatile int* verdict = reinterpret_cast<volatile int*>(tmem_slot + 1);
     ChunkIter pf;  // residual prefetch iterator (elected thread only)
     pf.init(tiles);
-    long loads = 0, consumed = 0;
+    long loads = 0, consumed = 0, stored = 0;
     if constexpr (TR::resid) {
       if (elected) {
         for (int e = 0; e < E && pf.valid; ++e) {
@@ -317,14 +322,16 @@ __global__ void __launch_bounds__(THREADS, 1)
           ++consumed;
         }
         {
-          // this thread: row r, columns [g*HW, g*HW + HW) of the chunk = 16-byte
-          // chunks 4g .. 4g+3 of the 128-byte staging row
+          // this thread: row r, columns [g*HW, g*HW + HW) of the chunk = the
+          // 16-byte pieces NC*g .. NC*g + NC-1 of the 128-byte staging row
           uint32_t v[HW];
           if (nk > 0) {
             if constexpr (HW == 32)
               tmem_ld_32x32b_x32(acc_tm + c * CW + g * HW, v);
-            else
+            else if constexpr (HW == 16)
               tmem_ld_16(acc_tm + c * CW + g * HW, v);
+            else
+              tmem_ld_8(acc_tm + c * CW + g * HW, v);
             tmem_ld_wait();
           } else {
 #pragma unroll
@@ -337,10 +344,10 @@ __global__ void __launch_bounds__(THREADS, 1)
           float bb[HW];
           load_bias<HW>(args.bias, n0 + c * CW + g * HW, N, bb);
           if constexpr (TR::f32) {
-            // 16 fp32; X_old arrived by TMA into the same swizzled row
+            // X_old arrived by TMA into the same swizzled row
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              float4* p = reinterpret_cast<float4*>(rowp + (((4 * g + j) ^ (r & 7)) << 4));
+            for (int j = 0; j < NC; ++j) {
+              float4* p = reinterpret_cast<float4*>(rowp + (((NC * g + j) ^ (r & 7)) << 4));
               float4 o = *p;
               o.x += __uint_as_float(v[4 * j]) + bb[4 * j];
               o.y += __uint_as_float(v[4 * j + 1]) + bb[4 * j + 1];
@@ -349,9 +356,8 @@ __global__ void __launch_bounds__(THREADS, 1)
               *p = o;
             }
           } else {
-            // 32 bf16
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
+            for (int j = 0; j < NC; ++j) {
               uint4 pk;
               pk.x = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 0]) + bb[8 * j + 0]),
                                  epi_act<EPI>(__uint_as_float(v[8 * j + 1]) + bb[8 * j + 1]));
@@ -361,24 +367,29 @@ __global__ void __launch_bounds__(THREADS, 1)
                                  epi_act<EPI>(__uint_as_float(v[8 * j + 5]) + bb[8 * j + 5]));
               pk.w = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 6]) + bb[8 * j + 6]),
                                  epi_act<EPI>(__uint_as_float(v[8 * j + 7]) + bb[8 * j + 7]));
-              *reinterpret_cast<uint4*>(rowp + (((4 * g + j) ^ (r & 7)) << 4)) = pk;
+              *reinterpret_cast<uint4*>(rowp + (((NC * g + j) ^ (r & 7)) << 4)) = pk;
             }
           }
         }
         fence_async_smem();
+        // The previous chunk's store (issued a whole chunk ago) must have read
+        // its buffer before anyone passes this barrier: after it, that buffer
+        // is written by the next chunk (E = 2) or refilled by the prefetch.
+        if (elected) bulk_wait_read_all();
         named_bar_sync(1, EPI_THREADS);
         if (elected) {
           tma_store_2d(&tmC, buf, n0 + c * CW, m0);
-          bulk_commit();
-          bulk_wait_read_all();  // buffer e may be refilled
+          bulk_commit();  // stays in flight while the next chunk is computed
           if constexpr (TR::resid) {
-            if (pf.valid) {
-              mbar_expect_tx(&rfull[e], CBUF);
-              tma_load_2d(buf, &tmC, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
+            if (stored > 0 && pf.valid) {
+              const int ep = e == 0 ? E - 1 : e - 1;  // buffer of the previous chunk
+              mbar_expect_tx(&rfull[ep], CBUF);
+              tma_load_2d(sC + ep * CBUF, &tmC, &rfull[ep], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
               pf.advance(tiles, nt, bn, CW, N);
               ++loads;
             }
           }
+          ++stored;
         }
         if (++e == E) {
           e = 0;
