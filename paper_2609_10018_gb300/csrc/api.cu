@@ -270,7 +270,8 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   const size_t rows = size_t(Bm) * n;
   const size_t o_X = bump.take(rows * D * 4), o_Y = bump.take(rows * D * 2);
   const size_t o_QKV = bump.take(rows * 3 * std::max(wmax, 64) * 2), o_O = bump.take(rows * std::max(wmax, 64) * 2);
-  const size_t o_H = bump.take(rows * std::max(fmax, 8) * 2), o_P = bump.take(size_t(Bm) * np * kpe * 2);
+  const size_t o_H = bump.take(rows * std::max(fmax, 8) * 2), o_P = bump.take(rows * kpe * 2);
+  const size_t o_tok = bump.take(rows * D * 4);  // per-token addend of the patch projection
   const size_t img_bytes = size_t(Bm) * d->img_h * d->img_w * d->img_c * dtype_size(d->weight_dtype);
   const size_t o_img = bump.take(img_bytes), o_logit = bump.take(size_t(Bm) * C * 4);
   const size_t o_status = bump.take(64);
@@ -307,6 +308,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   h->O = reinterpret_cast<bf16*>(A + o_O);
   h->H = reinterpret_cast<bf16*>(A + o_H);
   h->P = reinterpret_cast<bf16*>(A + o_P);
+  h->tok_addend = reinterpret_cast<float*>(A + o_tok);
   h->img_stage = A + o_img;
   h->logit_stage = reinterpret_cast<float*>(A + o_logit);
   h->status = reinterpret_cast<int*>(A + o_status);
@@ -453,11 +455,15 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
 
   // ---------------------------------------------------------------- plans
   const int Mcap = Bm * n;
-  st = gemm_plan(&h->patch, h->P, Bm * np, h->patch_w, D, kpe, h->patch_b, h->X, D, EPI_PATCH_POS_F32, h->status);
+  // Patch projection over token-ordered rows (class-token slots are zero
+  // rows): X = addend + P W_pe^T, addend = cls + pos[0] on class tokens and
+  // pos[t] + b_pe on patch tokens (Section 4.1: N = HW/P^2 patches, n = N + 1).
+  ELASTO_CUDA_TRY(token_addend_launch(h->cls, h->pos, h->patch_b, n, D, Bm, h->tok_addend, 0));
+  st = gemm_plan(&h->patch, h->P, Mcap, h->patch_w, D, kpe, nullptr, h->X, D, EPI_BIAS_RESID_F32, h->status);
   if (st != ELASTO_OK) return st;
-  h->patch.args.patches = np;
-  h->patch.args.tokens = n;
-  h->patch.args.pos = h->pos;
+  st = gemm_set_residual_source(&h->patch, h->tok_addend, Mcap);
+  if (st != ELASTO_OK) return st;
+  ELASTO_CUDA_TRY(cudaDeviceSynchronize());
   const int64_t lin_patch = int64_t(np) * D * kpe + int64_t(D) * C;
   for (int m = 0; m < n_modes; ++m) {
     VitMode& vm = h->modes[m];
@@ -525,11 +531,9 @@ elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int b
   const int n = h->n, D = d.dim, M = batch * n, Mp = batch * h->np, C = d.classes;
   const double img_elt = d.weight_dtype == ELASTO_BF16 ? 2 : 4;
   h->prof.begin();
-  ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, Mp, h->kpe, 0, 0,
-                         double(Mp) * h->kpe * (img_elt + 2) + double(batch) * D * 4),
-                patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, h->X, h->cls,
-                                h->pos, D, s));
-  ELASTO_LAUNCH(gemm_rec(-1, Mp, D, h->kpe, 4, false), gemm_launch(h->patch, Mp, s));
+  ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, M, h->kpe, 0, 0, double(Mp) * h->kpe * img_elt + double(M) * h->kpe * 2),
+                patch_rows_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, s));
+  ELASTO_LAUNCH(gemm_rec(-1, M, D, h->kpe, 4, true), gemm_launch(h->patch, M, s));
   const double ln_bytes = double(M) * D * (4 + 2);
   for (int l = 0; l < d.layers; ++l) {
     const VitLayerPack& lp = vm.layers[l];

@@ -67,6 +67,7 @@ struct GemmArgs {
 struct GemmPlan {
   CUtensorMap tmA, tmB;
   CUtensorMap tmC;        // output [M_cap, ldo] (bf16 or fp32), box 128 B x 128 rows, 128B swizzle
+  CUtensorMap tmR;        // residual source of EPI_BIAS_RESID_F32 (the output itself by default)
   GemmArgs args;          // M here is the capacity the A map was encoded for
   int epi = 0;
   bool valid = false;
@@ -78,6 +79,9 @@ int gemm_pick_bn(int M, int N, int step = 32);
 // allocated for the plan's life.
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
                         void* out, int ldo, int epi, int* status);
+// Residual epilogue: read the addend from src [M_cap, ldo] fp32 instead of
+// the output (out = src + acc + bias).
+elasto_status gemm_set_residual_source(GemmPlan* p, const float* src, int M_cap);
 // Launch for the first M (<= M_cap) rows.
 cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s);
 cudaError_t gemm_init_attributes();
@@ -103,6 +107,15 @@ cudaError_t softmax_launch(const float* x, float* y, int rows, int cols, cudaStr
 // order; also writes the class-token rows X[b * n] = cls + pos[0].
 cudaError_t patchify_launch(const void* images, int img_dtype, int B, int H, int W, int C, int P, bf16* A,
                             float* X, const float* cls, const float* pos, int d, cudaStream_t s);
+// images [B, H, W, C] -> A [B * n, P*P*C] bf16 in token order: row b*n is the
+// class token's slot (zeros), row b*n + 1 + p holds patch p in (ky, kx, c)
+// order. 16-byte copies when the images are bf16 and P*C % 8 == 0.
+cudaError_t patch_rows_launch(const void* images, int img_dtype, int B, int H, int W, int C, int P, bf16* A,
+                              cudaStream_t s);
+// dst [B * n, d] fp32 = the per-token addend of the patch projection, tiled
+// over the batch: row 0 of an image = cls + pos[0], row t >= 1 = pos[t] + b_pe.
+cudaError_t token_addend_launch(const float* cls, const float* pos, const float* patch_b, int n, int d, int B,
+                                float* dst, cudaStream_t s);
 // logits[b, c] = LN(X[b * n, :]) . head_w[c, :] + head_b[c], all fp32.
 cudaError_t head_launch(const float* X, int B, int n, int d, const float* g, const float* b, const float* Wh,
                         const float* bh, int C, float* logits, cudaStream_t s);

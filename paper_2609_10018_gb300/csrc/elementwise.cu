@@ -227,6 +227,95 @@ cudaError_t patchify_launch(const void* images, int img_dtype, int B, int H, int
   return cudaGetLastError();
 }
 
+namespace {
+
+// A [B * n, K] in token order, K = P*P*C in (ky, kx, c) order. One thread per
+// 16-byte piece (8 bf16): within a patch row, the P*C values (kx, c) are
+// contiguous in the NHWC image, so a piece is one aligned 16-byte copy.
+__global__ void patch_rows_vec_kernel(const bf16* __restrict__ img, int B, int H, int W, int C, int P,
+                                      uint4* __restrict__ A) {
+  const int gw = W / P, np = (H / P) * gw, n = np + 1, K = P * P * C;
+  const int row_pieces = K / 8, seg = P * C / 8;  // pieces per A row, per patch row
+  const size_t total = static_cast<size_t>(B) * n * row_pieces;
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const int j = static_cast<int>(t % row_pieces);
+    const size_t row = t / row_pieces;
+    const int tok = static_cast<int>(row % n), bb = static_cast<int>(row / n);
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (tok > 0) {
+      const int p = tok - 1, ky = j / seg, jj = j - ky * seg;
+      const int yy = (p / gw) * P + ky, x0 = (p % gw) * P;
+      v = *reinterpret_cast<const uint4*>(img + ((static_cast<size_t>(bb) * H + yy) * W + x0) * C + jj * 8);
+    }
+    A[t] = v;
+  }
+}
+
+// Generic version (fp32 images or P*C not a multiple of 8): one thread per element.
+template <typename T>
+__global__ void patch_rows_kernel(const T* __restrict__ img, int B, int H, int W, int C, int P, bf16* __restrict__ A) {
+  const int gw = W / P, np = (H / P) * gw, n = np + 1, K = P * P * C;
+  const size_t total = static_cast<size_t>(B) * n * K;
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const int k = static_cast<int>(t % K);
+    const size_t row = t / K;
+    const int tok = static_cast<int>(row % n), bb = static_cast<int>(row / n);
+    float v = 0.0f;
+    if (tok > 0) {
+      const int p = tok - 1, c = k % C, kx = (k / C) % P, ky = k / (C * P);
+      const T val = img[((static_cast<size_t>(bb) * H + (p / gw) * P + ky) * W + (p % gw) * P + kx) * C + c];
+      if constexpr (sizeof(T) == 2)
+        v = __bfloat162float(val);
+      else
+        v = static_cast<float>(val);
+    }
+    A[t] = __float2bfloat16_rn(v);
+  }
+}
+
+__global__ void token_addend_kernel(const float* __restrict__ cls, const float* __restrict__ pos,
+                                    const float* __restrict__ pb, int n, int d, size_t total, float* __restrict__ dst) {
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const int c = static_cast<int>(t % d);
+    const int tok = static_cast<int>((t / d) % n);
+    dst[t] = tok == 0 ? cls[c] + pos[c] : pos[static_cast<size_t>(tok) * d + c] + pb[c];
+  }
+}
+
+unsigned grid_1d(size_t n) {
+  const size_t b = (n + 255) / 256;
+  return static_cast<unsigned>(b < 16384 ? (b > 0 ? b : 1) : 16384);
+}
+
+}  // namespace
+
+cudaError_t patch_rows_launch(const void* images, int img_dtype, int B, int H, int W, int C, int P, bf16* A,
+                              cudaStream_t s) {
+  const int n = (H / P) * (W / P) + 1, K = P * P * C;
+  if (img_dtype == ELASTO_BF16 && (P * C) % 8 == 0) {
+    const size_t total = static_cast<size_t>(B) * n * (K / 8);
+    patch_rows_vec_kernel<<<grid_1d(total), 256, 0, s>>>(static_cast<const bf16*>(images), B, H, W, C, P,
+                                                         reinterpret_cast<uint4*>(A));
+  } else if (img_dtype == ELASTO_BF16) {
+    patch_rows_kernel<bf16><<<grid_1d(static_cast<size_t>(B) * n * K), 256, 0, s>>>(
+        static_cast<const bf16*>(images), B, H, W, C, P, A);
+  } else {
+    patch_rows_kernel<float><<<grid_1d(static_cast<size_t>(B) * n * K), 256, 0, s>>>(
+        static_cast<const float*>(images), B, H, W, C, P, A);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t token_addend_launch(const float* cls, const float* pos, const float* patch_b, int n, int d, int B,
+                                float* dst, cudaStream_t s) {
+  const size_t total = static_cast<size_t>(B) * n * d;
+  token_addend_kernel<<<grid_1d(total), 256, 0, s>>>(cls, pos, patch_b, n, d, total, dst);
+  return cudaGetLastError();
+}
+
 // ---------------------------------------------------------------- classifier
 namespace {
 

@@ -124,7 +124,8 @@ struct ChunkIter {
 template <int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmC, const GemmArgs args) {
+                   const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmR,
+                   const GemmArgs args) {
   using TR = EpiTraits<EPI>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -170,6 +171,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       tma_prefetch_desc(&tmB);
     }
     if constexpr (TR::tma) tma_prefetch_desc(&tmC);
+    if constexpr (TR::resid) tma_prefetch_desc(&tmR);
   }
   tc_fence_before();
   __syncthreads();
@@ -285,7 +287,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (elected) {
         for (int e = 0; e < E && pf.valid; ++e) {
           mbar_expect_tx(&rfull[e], CBUF);
-          tma_load_2d(sC + e * CBUF, &tmC, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
+          tma_load_2d(sC + e * CBUF, &tmR, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
           pf.advance(tiles, nt, bn, CW, N);
           ++loads;
         }
@@ -384,7 +386,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (stored > 0 && pf.valid) {
               const int ep = e == 0 ? E - 1 : e - 1;  // buffer of the previous chunk
               mbar_expect_tx(&rfull[ep], CBUF);
-              tma_load_2d(sC + ep * CBUF, &tmC, &rfull[ep], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
+              tma_load_2d(sC + ep * CBUF, &tmR, &rfull[ep], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
               pf.advance(tiles, nt, bn, CW, N);
               ++loads;
             }
@@ -506,7 +508,7 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   a.M = M;
   const int tiles = ((M + BM - 1) / BM) * ((a.N + a.bn - 1) / a.bn);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmC, a);
+  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmC, p.tmR, a);
   return cudaGetLastError();
 }
 
@@ -584,6 +586,7 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
       set_error("gemm_plan: output tensor map (alignment or size)");
       return ELASTO_ERR_UNSUPPORTED;
     }
+    p->tmR = p->tmC;  // the residual is read from the output unless redirected
   } else {
     a.stages = MAX_STAGES;
     a.cbufs = 0;
@@ -596,6 +599,19 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     }
   }
   p->valid = true;
+  return ELASTO_OK;
+}
+
+elasto_status gemm_set_residual_source(GemmPlan* p, const float* src, int M_cap) {
+  if (!p || !p->valid || p->epi != EPI_BIAS_RESID_F32 || !src) {
+    set_error("gemm_set_residual_source: needs a residual plan and a source");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int ldo = p->args.ldo;
+  if (!encode_tmap_2d(&p->tmR, src, ldo, M_cap, static_cast<uint64_t>(ldo) * 4, 32, BM, true)) {
+    set_error("gemm_set_residual_source: tensor map (alignment or size)");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
   return ELASTO_OK;
 }
 

@@ -46,6 +46,7 @@ struct elasto_s {
   // workspace
   float* X = nullptr;
   elasto::bf16 *Y = nullptr, *QKV = nullptr, *O = nullptr, *H = nullptr, *P = nullptr;
+  float* tok_addend = nullptr;  // [max_batch * n, d] addend of the patch projection
   void* img_stage = nullptr;
   float* logit_stage = nullptr;
   int* status = nullptr;
