@@ -241,8 +241,11 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   h->shared_bytes = bump.off;
 
   h->modes.assign(n_modes, VitMode{});
+  // fp32-stored models keep each weight as a bf16 pair (hi, lo): ~16 mantissa bits
+  const bool split = d->weight_dtype == ELASTO_F32;
   struct Off {
     size_t qkv_w, qkv_b, proj_w, fc1_w, fc1_b, fc2_w;
+    size_t qkv_lo = 0, proj_lo = 0, fc1_lo = 0, fc2_lo = 0;
   };
   std::vector<std::vector<Off>> offs(n_modes, std::vector<Off>(L));
   int wmax = 0, fmax = 0;
@@ -263,9 +266,16 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       o.fc1_w = bump.take(size_t(lp.f_pad) * D * 2);
       o.fc1_b = bump.take(size_t(lp.f_pad) * 4);
       o.fc2_w = bump.take(size_t(D) * lp.f_pad * 2);
+      if (split) {
+        o.qkv_lo = bump.take(size_t(3) * lp.w * D * 2);
+        o.proj_lo = bump.take(size_t(D) * lp.w * 2);
+        o.fc1_lo = bump.take(size_t(lp.f_pad) * D * 2);
+        o.fc2_lo = bump.take(size_t(D) * lp.f_pad * 2);
+      }
     }
     h->modes[m].packed_bytes = bump.off - start;
   }
+  const size_t o_patch_lo = split ? bump.take(size_t(D) * kpe * 2) : 0;
   const size_t ws_start = bump.off;
   const size_t rows = size_t(Bm) * n;
   const size_t o_X = bump.take(rows * D * 4), o_Y = bump.take(rows * D * 2);
@@ -287,6 +297,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   }
   char* A = h->arena;
   h->patch_w = reinterpret_cast<bf16*>(A + o_patch_w);
+  h->patch_w_lo = split ? reinterpret_cast<bf16*>(A + o_patch_lo) : nullptr;
   h->patch_b = reinterpret_cast<float*>(A + o_patch_b);
   h->cls = reinterpret_cast<float*>(A + o_cls);
   h->pos = reinterpret_cast<float*>(A + o_pos);
@@ -322,6 +333,12 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       lp.fc1_w = reinterpret_cast<bf16*>(A + o.fc1_w);
       lp.fc1_b = reinterpret_cast<float*>(A + o.fc1_b);
       lp.fc2_w = reinterpret_cast<bf16*>(A + o.fc2_w);
+      if (split) {
+        lp.qkv_w_lo = reinterpret_cast<bf16*>(A + o.qkv_lo);
+        lp.proj_w_lo = reinterpret_cast<bf16*>(A + o.proj_lo);
+        lp.fc1_w_lo = reinterpret_cast<bf16*>(A + o.fc1_lo);
+        lp.fc2_w_lo = reinterpret_cast<bf16*>(A + o.fc2_lo);
+      }
     }
   ELASTO_CUDA_TRY(cudaMemset(h->arena, 0, h->arena_bytes));
 
@@ -331,9 +348,10 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   auto W = [&](int i) { return wts->tensors[i]; };
   // temp: raw upload buffer + canonical bf16 + canonical fp32 bias + index list
   const size_t max_mat = std::max({size_t(3) * D * D, size_t(F) * D, size_t(D) * kpe});
-  DevTemp raw, canon, canon_b, idxbuf;
+  DevTemp raw, canon, canon_lo, canon_b, idxbuf;
   ELASTO_CUDA_TRY(cudaMalloc(&raw.p, max_mat * 4 + size_t(n) * D * 4 + size_t(C) * D * 4));
   ELASTO_CUDA_TRY(cudaMalloc(&canon.p, max_mat * 2));
+  if (split) ELASTO_CUDA_TRY(cudaMalloc(&canon_lo.p, max_mat * 2));
   ELASTO_CUDA_TRY(cudaMalloc(&canon_b.p, size_t(std::max(3 * D, F)) * 4));
   ELASTO_CUDA_TRY(cudaMalloc(&idxbuf.p, size_t(std::max(3 * D, F) + 64) * 4));
   cudaStream_t s = 0;
@@ -368,6 +386,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
             memcpy(re.data() + di * es, src + si * es, es);
           }
     UP(up_bf16(re.data(), size_t(D) * kpe, h->patch_w));
+    if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(D) * kpe, h->patch_w_lo, s));
   }
   UP(up_f32(W(1), D, h->patch_b));
   UP(up_f32(W(2), D, h->cls));
@@ -388,10 +407,12 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     UP(up_f32(W(t0 + 7), D, h->ln2_b[l]));
     UP(up_f32(W(t0 + 11), D, h->fc2_b[l]));
     bf16* cw = static_cast<bf16*>(canon.p);
+    bf16* cwl = static_cast<bf16*>(canon_lo.p);
     float* cb = static_cast<float*>(canon_b.p);
     int32_t* di = static_cast<int32_t*>(idxbuf.p);
     // qkv: rows {blk * d + j * 64 + r}
     UP(up_bf16(W(t0 + 2), size_t(3) * D * D, cw));
+    if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(3) * D * D, cwl, s));
     UP(up_f32(W(t0 + 3), size_t(3) * D, cb));
     for (int m = 0; m < n_modes; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
@@ -405,11 +426,13 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
           for (int r = 0; r < 64; ++r) idx.push_back(blk * D + hk[j] * 64 + r);
       ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
       ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, int(idx.size()), lp.qkv_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, int(idx.size()), lp.qkv_w_lo, s));
       ELASTO_CUDA_TRY(gather_f32(cb, di, int(idx.size()), lp.qkv_b, s));
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
     // proj: columns {j * 64 + r}
     UP(up_bf16(W(t0 + 4), size_t(D) * D, cw));
+    if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(D) * D, cwl, s));
     for (int m = 0; m < n_modes; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
       if (lp.w == 0) continue;
@@ -421,10 +444,12 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
         for (int r = 0; r < 64; ++r) idx.push_back(hk[j] * 64 + r);
       ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
       ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, D, di, int(idx.size()), lp.proj_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, D, di, int(idx.size()), lp.proj_w_lo, s));
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
     // fc1: rows F (padding rows stay zero), b1 entries F
     UP(up_bf16(W(t0 + 8), size_t(F) * D, cw));
+    if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(F) * D, cwl, s));
     UP(up_f32(W(t0 + 9), F, cb));
     for (int m = 0; m < n_modes; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
@@ -433,11 +458,13 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       for (int k = 0; k < l; ++k) fo += modes[m].n_mlp_kept[k];
       ELASTO_CUDA_TRY(cudaMemcpy(di, modes[m].mlp_kept + fo, size_t(lp.f) * 4, cudaMemcpyHostToDevice));
       ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, lp.f, lp.fc1_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, lp.f, lp.fc1_w_lo, s));
       ELASTO_CUDA_TRY(gather_f32(cb, di, lp.f, lp.fc1_b, s));
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
     // fc2: columns F into [d, f_pad] (padding columns zero)
     UP(up_bf16(W(t0 + 10), size_t(D) * F, cw));
+    if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(D) * F, cwl, s));
     for (int m = 0; m < n_modes; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
       if (lp.f == 0) continue;
@@ -447,6 +474,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       for (int k = lp.f; k < lp.f_pad; ++k) idx.push_back(-1);
       ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
       ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, F, di, lp.f_pad, lp.fc2_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, F, di, lp.f_pad, lp.fc2_w_lo, s));
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
   }
@@ -459,7 +487,8 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   // rows): X = addend + P W_pe^T, addend = cls + pos[0] on class tokens and
   // pos[t] + b_pe on patch tokens (Section 4.1: N = HW/P^2 patches, n = N + 1).
   ELASTO_CUDA_TRY(token_addend_launch(h->cls, h->pos, h->patch_b, n, D, Bm, h->tok_addend, 0));
-  st = gemm_plan(&h->patch, h->P, Mcap, h->patch_w, D, kpe, nullptr, h->X, D, EPI_BIAS_RESID_F32, h->status);
+  st = gemm_plan(&h->patch, h->P, Mcap, h->patch_w, D, kpe, nullptr, h->X, D, EPI_BIAS_RESID_F32, h->status,
+                 h->patch_w_lo);
   if (st != ELASTO_OK) return st;
   st = gemm_set_residual_source(&h->patch, h->tok_addend, Mcap);
   if (st != ELASTO_OK) return st;
@@ -476,21 +505,23 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       vm.launches += 2;  // two LayerNorms
       if (lp.w > 0) {
         st = gemm_plan(&lp.qkv, h->Y, Mcap, lp.qkv_w, 3 * lp.w, D, lp.qkv_b, h->QKV, 3 * lp.w, EPI_BIAS_BF16,
-                       h->status);
+                       h->status, lp.qkv_w_lo);
         if (st != ELASTO_OK) return st;
         st = attn_plan(&lp.attn, h->QKV, h->O, Bm, n, lp.w / 64, h->status);
         if (st != ELASTO_OK) return st;
         vm.launches += 2;
       }
-      st = gemm_plan(&lp.proj, h->O, Mcap, lp.proj_w, D, lp.w, h->proj_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status);
+      st = gemm_plan(&lp.proj, h->O, Mcap, lp.proj_w, D, lp.w, h->proj_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
+                     lp.proj_w_lo);
       if (st != ELASTO_OK) return st;
       if (lp.f > 0) {
         st = gemm_plan(&lp.fc1, h->Y, Mcap, lp.fc1_w, lp.f_pad, D, lp.fc1_b, h->H, lp.f_pad, EPI_BIAS_GELU_BF16,
-                       h->status);
+                       h->status, lp.fc1_w_lo);
         if (st != ELASTO_OK) return st;
         vm.launches += 1;
       }
-      st = gemm_plan(&lp.fc2, h->H, Mcap, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status);
+      st = gemm_plan(&lp.fc2, h->H, Mcap, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
+                     lp.fc2_w_lo);
       if (st != ELASTO_OK) return st;
       vm.launches += 2;
     }

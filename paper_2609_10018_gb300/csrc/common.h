@@ -62,10 +62,11 @@ struct GemmArgs {
   int* status;
   int stages;             // operand ring depth (<= 4)
   int cbufs;              // output staging buffers (16 KB each) for the TMA-store epilogues
+  int b_planes;           // 2: W held as bf16 hi + lo planes (fp32-stored models), both multiplied
 };
 
 struct GemmPlan {
-  CUtensorMap tmA, tmB;
+  CUtensorMap tmA, tmB, tmB2;  // tmB2: low bf16 plane of W (b_planes == 2)
   CUtensorMap tmC;        // output [M_cap, ldo] (bf16 or fp32), box 128 B x 128 rows, 128B swizzle
   CUtensorMap tmR;        // residual source of EPI_BIAS_RESID_F32 (the output itself by default)
   GemmArgs args;          // M here is the capacity the A map was encoded for
@@ -77,8 +78,10 @@ struct GemmPlan {
 int gemm_pick_bn(int M, int N, int step = 32);
 // Build maps/arguments for out = epi(A[M_cap, K] W[N, K]^T). A and W must stay
 // allocated for the plan's life.
+// W_lo (optional): second bf16 plane so that W = W + W_lo carries ~16
+// mantissa bits (used for models stored in fp32); both products accumulate.
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
-                        void* out, int ldo, int epi, int* status);
+                        void* out, int ldo, int epi, int* status, const bf16* W_lo = nullptr);
 // Residual epilogue: read the addend from src [M_cap, ldo] fp32 instead of
 // the output (out = src + acc + bias).
 elasto_status gemm_set_residual_source(GemmPlan* p, const float* src, int M_cap);
@@ -125,6 +128,8 @@ cudaError_t gather_cols_bf16(const bf16* src, int rows, int cols, const int32_t*
                              cudaStream_t s);
 cudaError_t gather_f32(const float* src, const int32_t* idx, int nidx, float* dst, cudaStream_t s);
 cudaError_t convert_to_bf16(const void* src, int src_dtype, size_t n, bf16* dst, cudaStream_t s);
+// dst = bf16(x - bf16(x)) for fp32 sources (the low plane of a bf16 pair); zeros for bf16 sources.
+cudaError_t convert_to_bf16_lo(const void* src, int src_dtype, size_t n, bf16* dst, cudaStream_t s);
 cudaError_t convert_to_f32(const void* src, int src_dtype, size_t n, float* dst, cudaStream_t s);
 
 }  // namespace elasto

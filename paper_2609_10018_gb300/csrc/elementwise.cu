@@ -466,6 +466,23 @@ cudaError_t convert_to_bf16(const void* src, int src_dtype, size_t n, bf16* dst,
     to_bf16_kernel<float><<<grid_for(n), 256, 0, s>>>(static_cast<const float*>(src), n, dst);
   return cudaGetLastError();
 }
+namespace {
+__global__ void to_bf16_lo_kernel(const float* __restrict__ src, size_t n, bf16* __restrict__ dst) {
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < n;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const float x = src[t];
+    dst[t] = __float2bfloat16_rn(x - __bfloat162float(__float2bfloat16_rn(x)));
+  }
+}
+}  // namespace
+
+cudaError_t convert_to_bf16_lo(const void* src, int src_dtype, size_t n, bf16* dst, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  if (src_dtype == ELASTO_BF16) return cudaMemsetAsync(dst, 0, n * sizeof(bf16), s);
+  to_bf16_lo_kernel<<<grid_for(n), 256, 0, s>>>(static_cast<const float*>(src), n, dst);
+  return cudaGetLastError();
+}
+
 cudaError_t convert_to_f32(const void* src, int src_dtype, size_t n, float* dst, cudaStream_t s) {
   if (n == 0) return cudaSuccess;
   if (src_dtype == ELASTO_BF16)

@@ -121,9 +121,10 @@ struct ChunkIter {
   }
 };
 
-template <int EPI>
+template <int EPI, int NB>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmB2,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmR,
                    const GemmArgs args) {
   using TR = EpiTraits<EPI>;
@@ -132,7 +133,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int S = args.stages, E = args.cbufs;
   uint8_t* sA = smem;
   uint8_t* sB = smem + S * A_STAGE;
-  uint8_t* sC = sB + S * B_STAGE;  // E staging chunks, or the transpose tiles
+  // NB: 1, or 2 when W is held as a bf16 (hi, lo) pair
+  uint8_t* sC = sB + S * NB * B_STAGE;  // E staging chunks, or the transpose tiles
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + POOL);
   uint64_t* full = bars;
   uint64_t* empty = bars + MAX_STAGES;
@@ -169,6 +171,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (nk > 0) {
       tma_prefetch_desc(&tmA);
       tma_prefetch_desc(&tmB);
+      if constexpr (NB == 2) tma_prefetch_desc(&tmB2);
     }
     if constexpr (TR::tma) tma_prefetch_desc(&tmC);
     if constexpr (TR::resid) tma_prefetch_desc(&tmR);
@@ -185,7 +188,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t phase = 0;
       long issued = 0;
       bool ok = true;
-      const uint32_t bytes = A_STAGE + bn * BK * 2;
+      const uint32_t bytes = A_STAGE + NB * bn * BK * 2;
       for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
         const int m0 = (t / nt) * BM, n0 = (t % nt) * bn;
         for (int kb = 0; kb < nk; ++kb) {
@@ -195,7 +198,8 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           mbar_expect_tx(&full[stage], bytes);
           tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
-          tma_load_2d(sB + stage * B_STAGE, &tmB, &full[stage], kb * BK, n0);
+          tma_load_2d(sB + stage * NB * B_STAGE, &tmB, &full[stage], kb * BK, n0);
+          if constexpr (NB == 2) tma_load_2d(sB + (stage * 2 + 1) * B_STAGE, &tmB2, &full[stage], kb * BK, n0);
           ++issued;
           if (++stage == S) {
             stage = 0;
@@ -242,11 +246,14 @@ __global__ void __launch_bounds__(THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_addr(sA + stage * A_STAGE), b0 = smem_addr(sB + stage * B_STAGE);
+          const uint32_t a0 = smem_addr(sA + stage * A_STAGE), b0 = smem_addr(sB + stage * NB * B_STAGE);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
                    (kb | k) != 0);
+            if constexpr (NB == 2)  // low half of the weights: acc += A . W_lo^T
+              tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + B_STAGE + k * 32, 16, 1024), idesc,
+                     1u);
           }
           issued = true;
           tc_commit(&empty[stage]);
@@ -502,13 +509,13 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
-template <int EPI>
+template <int EPI, int NB>
 cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   GemmArgs a = p.args;
   a.M = M;
   const int tiles = ((M + BM - 1) / BM) * ((a.N + a.bn - 1) / a.bn);
   const int grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_tc_kernel<EPI><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmC, p.tmR, a);
+  gemm_tc_kernel<EPI, NB><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
   return cudaGetLastError();
 }
 
@@ -518,7 +525,9 @@ cudaError_t gemm_init_attributes() {
   const int bytes = static_cast<int>(SMEM_BYTES);
   cudaError_t e;
 #define SET_ATTR(E)                                                                                     \
-  e = cudaFuncSetAttribute(gemm_tc_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);      \
+  e = cudaFuncSetAttribute(gemm_tc_kernel<E, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);   \
+  if (e != cudaSuccess) return e;                                                                       \
+  e = cudaFuncSetAttribute(gemm_tc_kernel<E, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);   \
   if (e != cudaSuccess) return e;
   SET_ATTR(EPI_BIAS_BF16)
   SET_ATTR(EPI_BIAS_GELU_BF16)
@@ -550,7 +559,7 @@ int gemm_pick_bn(int M, int N, int step) {
 }
 
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
-                        void* out, int ldo, int epi, int* status) {
+                        void* out, int ldo, int epi, int* status, const bf16* W_lo) {
   if (!p || M_cap <= 0 || N <= 0 || K < 0 || !out || (K > 0 && (!A || !W))) {
     set_error("gemm_plan: invalid arguments");
     return ELASTO_ERR_INVALID_ARG;
@@ -573,12 +582,13 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   a.out = out;
   a.ldo = ldo;
   a.status = status;
+  a.b_planes = W_lo ? 2 : 1;
   p->epi = epi;
   if (tma_out) {
     // residual GEMMs: 3 operand stages and 5 staging chunks fetched ahead;
     // the others: 4 stages and 2 staging chunks.
-    a.stages = f32_out ? 3 : 4;
-    a.cbufs = (POOL - a.stages * (A_STAGE + B_STAGE)) / CBUF;
+    a.stages = W_lo ? 2 : (f32_out ? 3 : 4);
+    a.cbufs = (POOL - a.stages * (A_STAGE + a.b_planes * B_STAGE)) / CBUF;
     if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
     if (ldo % 8 != 0 ||
         !encode_tmap_2d(&p->tmC, out, ldo, M_cap, static_cast<uint64_t>(ldo) * (f32_out ? 4 : 2),
@@ -588,12 +598,13 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     }
     p->tmR = p->tmC;  // the residual is read from the output unless redirected
   } else {
-    a.stages = MAX_STAGES;
+    a.stages = W_lo ? 2 : MAX_STAGES;
     a.cbufs = 0;
   }
   if (K > 0) {
     if (!encode_tmap_2d(&p->tmA, A, K, M_cap, static_cast<uint64_t>(K) * 2, BK, BM) ||
-        !encode_tmap_2d(&p->tmB, W, K, N, static_cast<uint64_t>(K) * 2, BK, a.bn)) {
+        !encode_tmap_2d(&p->tmB, W, K, N, static_cast<uint64_t>(K) * 2, BK, a.bn) ||
+        (W_lo && !encode_tmap_2d(&p->tmB2, W_lo, K, N, static_cast<uint64_t>(K) * 2, BK, a.bn))) {
       set_error("gemm_plan: cuTensorMapEncodeTiled failed (alignment or size)");
       return ELASTO_ERR_UNSUPPORTED;
     }
@@ -617,14 +628,18 @@ elasto_status gemm_set_residual_source(GemmPlan* p, const float* src, int M_cap)
 
 cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
+  const bool two = p.args.b_planes == 2;
+#define CASE(E) \
+  case E: return two ? launch_epi<E, 2>(p, M, s) : launch_epi<E, 1>(p, M, s);
   switch (p.epi) {
-    case EPI_BIAS_BF16: return launch_epi<EPI_BIAS_BF16>(p, M, s);
-    case EPI_BIAS_GELU_BF16: return launch_epi<EPI_BIAS_GELU_BF16>(p, M, s);
-    case EPI_BIAS_RESID_F32: return launch_epi<EPI_BIAS_RESID_F32>(p, M, s);
-    case EPI_BIAS_F32: return launch_epi<EPI_BIAS_F32>(p, M, s);
-    case EPI_BIAS_RELU_BF16: return launch_epi<EPI_BIAS_RELU_BF16>(p, M, s);
-    case EPI_BIAS_RESID_RELU_BF16: return launch_epi<EPI_BIAS_RESID_RELU_BF16>(p, M, s);
-    case EPI_PATCH_POS_F32: return launch_epi<EPI_PATCH_POS_F32>(p, M, s);
+    CASE(EPI_BIAS_BF16)
+    CASE(EPI_BIAS_GELU_BF16)
+    CASE(EPI_BIAS_RESID_F32)
+    CASE(EPI_BIAS_F32)
+    CASE(EPI_BIAS_RELU_BF16)
+    CASE(EPI_BIAS_RESID_RELU_BF16)
+    CASE(EPI_PATCH_POS_F32)
+#undef CASE
     default: return cudaErrorInvalidValue;
   }
 }

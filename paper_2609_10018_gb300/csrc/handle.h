@@ -19,6 +19,8 @@ struct VitLayerPack {
   bf16* fc1_w = nullptr;
   float* fc1_b = nullptr;
   bf16* fc2_w = nullptr;
+  // low bf16 planes (fp32-stored models only; W = hi + lo)
+  bf16 *qkv_w_lo = nullptr, *proj_w_lo = nullptr, *fc1_w_lo = nullptr, *fc2_w_lo = nullptr;
   GemmPlan qkv, proj, fc1, fc2;
   AttnPlan attn;
 };
@@ -40,6 +42,7 @@ struct elasto_s {
   size_t arena_bytes = 0, shared_bytes = 0, workspace_bytes = 0;
   // shared (mode-independent) parameters
   elasto::bf16* patch_w = nullptr;
+  elasto::bf16* patch_w_lo = nullptr;  // low plane for fp32-stored models
   float *patch_b = nullptr, *cls = nullptr, *pos = nullptr, *norm_w = nullptr, *norm_b = nullptr;
   float *head_w = nullptr, *head_b = nullptr;
   std::vector<float*> ln1_w, ln1_b, proj_b, ln2_w, ln2_b, fc2_b;

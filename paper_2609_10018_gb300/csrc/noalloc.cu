@@ -129,7 +129,8 @@ extern "C" elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const 
   const int n = h->n, D = d.dim, M = batch * n, Mp = batch * h->np;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   GemmPlan gp;
-  st = gemm_plan(&gp, P, Mp, h->patch_w, D, h->kpe, h->patch_b, X, D, EPI_PATCH_POS_F32, h->status);
+  st = gemm_plan(&gp, P, Mp, h->patch_w, D, h->kpe, h->patch_b, X, D, EPI_PATCH_POS_F32, h->status,
+                 h->patch_w_lo);
   if (st != ELASTO_OK) return st;
   gp.args.patches = h->np;
   gp.args.tokens = n;
@@ -144,27 +145,27 @@ extern "C" elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const 
       GemmPlan qkv;
       AttnPlan at;
       if ((st = gemm_plan(&qkv, Y, M, lp.qkv_w, 3 * lp.w, D, lp.qkv_b, QKV, 3 * lp.w, EPI_BIAS_BF16,
-                          h->status)) != ELASTO_OK)
+                          h->status, lp.qkv_w_lo)) != ELASTO_OK)
         return st;
       if ((st = attn_plan(&at, QKV, O, batch, n, lp.w / 64, h->status)) != ELASTO_OK) return st;
       ELASTO_CUDA_TRY(gemm_launch(qkv, M, s));
       ELASTO_CUDA_TRY(attn_launch(at, batch, s));
     }
     GemmPlan proj, fc2;
-    if ((st = gemm_plan(&proj, O, M, lp.proj_w, D, lp.w, h->proj_b[l], X, D, EPI_BIAS_RESID_F32, h->status)) !=
-        ELASTO_OK)
+    if ((st = gemm_plan(&proj, O, M, lp.proj_w, D, lp.w, h->proj_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
+                        lp.proj_w_lo)) != ELASTO_OK)
       return st;
     ELASTO_CUDA_TRY(gemm_launch(proj, M, s));
     ELASTO_CUDA_TRY(layernorm_launch(X, h->ln2_w[l], h->ln2_b[l], Y, M, D, s));
     if (lp.f > 0) {
       GemmPlan fc1;
       if ((st = gemm_plan(&fc1, Y, M, lp.fc1_w, lp.f_pad, D, lp.fc1_b, H, lp.f_pad, EPI_BIAS_GELU_BF16,
-                          h->status)) != ELASTO_OK)
+                          h->status, lp.fc1_w_lo)) != ELASTO_OK)
         return st;
       ELASTO_CUDA_TRY(gemm_launch(fc1, M, s));
     }
-    if ((st = gemm_plan(&fc2, H, M, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], X, D, EPI_BIAS_RESID_F32, h->status)) !=
-        ELASTO_OK)
+    if ((st = gemm_plan(&fc2, H, M, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
+                        lp.fc2_w_lo)) != ELASTO_OK)
       return st;
     ELASTO_CUDA_TRY(gemm_launch(fc2, M, s));
   }
