@@ -63,6 +63,7 @@ struct GemmArgs {
   int stages;             // operand ring depth (<= 4)
   int cbufs;              // output staging buffers (16 KB each) for the TMA-store epilogues
   int b_planes;           // 2: W held as bf16 hi + lo planes (fp32-stored models), both multiplied
+  int pair;               // 1: clusters of two CTAs sharing 256-row tiles (tcgen05 cta_group::2)
 };
 
 struct GemmPlan {
@@ -75,7 +76,7 @@ struct GemmPlan {
 };
 
 // Pick the N tile for an M x N problem.
-int gemm_pick_bn(int M, int N, int step = 32);
+int gemm_pick_bn(int M, int N, int step = 32, bool pair = false);
 // Build maps/arguments for out = epi(A[M_cap, K] W[N, K]^T). A and W must stay
 // allocated for the plan's life.
 // W_lo (optional): second bf16 plane so that W = W + W_lo carries ~16

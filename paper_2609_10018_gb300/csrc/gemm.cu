@@ -34,11 +34,12 @@ namespace elasto {
 
 namespace {
 
-constexpr int BM = 128, BK = 64, MAX_STAGES = 4, MAX_BN = 256;
+constexpr int BM = 128, BK = 64, MAX_STAGES = 8, MAX_BN = 256;
 constexpr int EPI_THREADS = 512;                 // 16 epilogue warps, four per TMEM lane quarter
 constexpr int THREADS = 64 + EPI_THREADS;
 constexpr int A_STAGE = BM * BK * 2;        // 16 KB
 constexpr int B_STAGE = MAX_BN * BK * 2;    // 32 KB
+constexpr int B_STAGE_PAIR = B_STAGE / 2;   // a CTA of a pair holds half of B
 constexpr int CBUF = BM * 128;              // 16 KB staging chunk (128 rows x 128 B)
 constexpr int POOL = 224 * 1024;            // operand ring + staging buffers
 constexpr int MAX_CBUFS = 8;
@@ -105,8 +106,10 @@ __device__ __forceinline__ void load_bias(const float* bias, int col, int N, flo
 struct ChunkIter {
   int t, c;
   bool valid;
-  __device__ __forceinline__ void init(int tiles) {
-    t = blockIdx.x;
+  int stride;
+  __device__ __forceinline__ void init(int tiles, int start, int step) {
+    t = start;
+    stride = step;
     c = 0;
     valid = t < tiles;
   }
@@ -115,13 +118,18 @@ struct ChunkIter {
     ++c;
     if (c * cw >= bn || n0 + c * cw >= N) {
       c = 0;
-      t += gridDim.x;
+      t += stride;
       valid = t < tiles;
     }
   }
 };
 
-template <int EPI, int NB>
+// PAIR: the kernel runs as clusters of two CTAs on neighbouring SMs that
+// share 256-row tiles: each CTA loads its 128 rows of A and half of the B
+// tile; the even CTA issues tcgen05.mma.cta_group::2 (M = 256) for both and
+// signals both CTAs' barriers with multicast commits; each CTA's epilogue
+// reads its own half of the accumulator from its own TMEM.
+template <int EPI, int NB, bool PAIR>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmB2,
@@ -131,10 +139,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = args.stages, E = args.cbufs;
+  // NB: 1, or 2 when W is held as a bf16 (hi, lo) pair
+  constexpr int BSTG = PAIR ? B_STAGE_PAIR : NB * B_STAGE;
   uint8_t* sA = smem;
   uint8_t* sB = smem + S * A_STAGE;
-  // NB: 1, or 2 when W is held as a bf16 (hi, lo) pair
-  uint8_t* sC = sB + S * NB * B_STAGE;  // E staging chunks, or the transpose tiles
+  uint8_t* sC = sB + S * BSTG;  // E staging chunks, or the transpose tiles
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + POOL);
   uint64_t* full = bars;
   uint64_t* empty = bars + MAX_STAGES;
@@ -147,8 +156,13 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int M = args.M, N = args.N, bn = args.bn;
   const int nk = (args.K + BK - 1) / BK;
-  const int mt = (M + BM - 1) / BM, nt = (N + bn - 1) / bn;
+  constexpr int TM = PAIR ? 2 * BM : BM;  // rows per tile
+  const int mt = (M + TM - 1) / TM, nt = (N + bn - 1) / bn;
   const int tiles = mt * nt;
+  const int rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;  // this CTA's row half of a pair tile
+  const int t_start = PAIR ? static_cast<int>(cluster_id_x()) : static_cast<int>(blockIdx.x);
+  const int t_stride = PAIR ? static_cast<int>(cluster_count_x()) : static_cast<int>(gridDim.x);
+  const bool leader = rank == 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < MAX_STAGES; ++s) {
@@ -157,15 +171,20 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&tfull[a], 1);
-      mbar_init(&tempty[a], TR::tma ? EPI_THREADS / 32 : 4);
+      mbar_init(&tempty[a], (PAIR ? 2 : 1) * (TR::tma ? EPI_THREADS / 32 : 4));
     }
     mbar_init(drain, 1);
     for (int e = 0; e < MAX_CBUFS; ++e) mbar_init(&rfull[e], 1);
     fence_barrier_init();
   }
   if (warp == 0) {
-    tmem_alloc(tmem_slot, TMEM_COLS);
-    tmem_relinquish();
+    if constexpr (PAIR) {
+      tmem_alloc_pair(tmem_slot, TMEM_COLS);
+      tmem_relinquish_pair();
+    } else {
+      tmem_alloc(tmem_slot, TMEM_COLS);
+      tmem_relinquish();
+    }
   }
   if (warp == 1 && lane == 0) {
     if (nk > 0) {
@@ -177,7 +196,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     if constexpr (TR::resid) tma_prefetch_desc(&tmR);
   }
   tc_fence_before();
-  __syncthreads();
+  if constexpr (PAIR)
+    cluster_sync_all();  // both CTAs' barriers initialised before any remote arrive
+  else
+    __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -188,18 +210,31 @@ __global__ void __launch_bounds__(THREADS, 1)
       uint32_t phase = 0;
       long issued = 0;
       bool ok = true;
-      const uint32_t bytes = A_STAGE + NB * bn * BK * 2;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x) {
-        const int m0 = (t / nt) * BM, n0 = (t % nt) * bn;
+      // pair: the even CTA's full barrier counts both CTAs' bytes
+      const uint32_t bytes = PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2) : A_STAGE + NB * bn * BK * 2;
+      for (int t = t_start; t < tiles && ok; t += t_stride) {
+        const int m0 = (t / nt) * TM + rank * BM, n0 = (t % nt) * bn;
         for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1)) {
+          if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
             ok = false;
             break;
           }
+          if constexpr (PAIR) {
+            const uint32_t full_lead = cluster_map(smem_addr(&full[stage]), 0);
+            if (leader) mbar_expect_tx(&full[stage], bytes);
+            tma_load_2d_pair(sA + stage * A_STAGE, &tmA, full_lead, kb * BK, m0);
+            tma_load_2d_pair(sB + stage * BSTG, &tmB, full_lead, kb * BK, n0 + rank * (bn / 2));
+            ++issued;
+            if (++stage == S) {
+              stage = 0;
+              phase ^= 1;
+            }
+            continue;
+          }
           mbar_expect_tx(&full[stage], bytes);
           tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
-          tma_load_2d(sB + stage * NB * B_STAGE, &tmB, &full[stage], kb * BK, n0);
-          if constexpr (NB == 2) tma_load_2d(sB + (stage * 2 + 1) * B_STAGE, &tmB2, &full[stage], kb * BK, n0);
+          tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * BK, n0);
+          if constexpr (NB == 2) tma_load_2d(sB + stage * BSTG + B_STAGE, &tmB2, &full[stage], kb * BK, n0);
           ++issued;
           if (++stage == S) {
             stage = 0;
@@ -209,28 +244,30 @@ __global__ void __launch_bounds__(THREADS, 1)
       }
       if (!ok) record_status(args.status, ELASTO_ERR_TIMEOUT);
       // Drain: no copy may still be landing in shared memory when the CTA
-      // exits (returns at once on the normal path).
-      for (int i = 0; i < S && i < issued; ++i) {
+      // exits (returns at once on the normal path). In a pair only the even
+      // CTA's barriers see the copies; the cluster barrier before exit
+      // orders the odd CTA behind this drain.
+      for (int i = 0; i < S && i < issued && leader; ++i) {
         if (stage == 0) {
           stage = S;
           phase ^= 1;
         }
         --stage;
-        mbar_wait(&full[stage], phase);
+        PAIR ? mbar_wait_cluster(&full[stage], phase) : mbar_wait(&full[stage], phase);
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      const uint32_t idesc = idesc_bf16_f32(BM, bn);
+    if (lane == 0 && leader) {
+      const uint32_t idesc = idesc_bf16_f32(TM, bn);
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true, issued = false;
       int local = 0;
-      for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++local) {
+      for (int t = t_start; t < tiles && ok; t += t_stride, ++local) {
         const int acc = local & 1;
         const uint32_t use = static_cast<uint32_t>(local >> 1);
-        if (!mbar_wait(&tempty[acc], (use & 1) ^ 1)) {
+        if (!(PAIR ? mbar_wait_cluster(&tempty[acc], (use & 1) ^ 1) : mbar_wait(&tempty[acc], (use & 1) ^ 1))) {
           ok = false;
           break;
         }
@@ -238,36 +275,53 @@ __global__ void __launch_bounds__(THREADS, 1)
         const uint32_t dtm = tmem_base + acc * MAX_BN;
         if (nk == 0) {
           mbar_arrive(&tfull[acc]);
+          if constexpr (PAIR) mbar_arrive_cluster(cluster_map(smem_addr(&tfull[acc]), 1));
           continue;
         }
         for (int kb = 0; kb < nk; ++kb) {
-          if (!mbar_wait(&full[stage], phase)) {
+          if (!(PAIR ? mbar_wait_cluster(&full[stage], phase) : mbar_wait(&full[stage], phase))) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_addr(sA + stage * A_STAGE), b0 = smem_addr(sB + stage * NB * B_STAGE);
+          const uint32_t a0 = smem_addr(sA + stage * A_STAGE), b0 = smem_addr(sB + stage * BSTG);
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
-            tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
-                   (kb | k) != 0);
-            if constexpr (NB == 2)  // low half of the weights: acc += A . W_lo^T
-              tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + B_STAGE + k * 32, 16, 1024), idesc,
-                     1u);
+            if constexpr (PAIR) {
+              tc_mma_pair(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
+                          (kb | k) != 0);
+            } else {
+              tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
+                     (kb | k) != 0);
+              if constexpr (NB == 2)  // low half of the weights: acc += A . W_lo^T
+                tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + B_STAGE + k * 32, 16, 1024),
+                       idesc, 1u);
+            }
           }
           issued = true;
-          tc_commit(&empty[stage]);
+          if constexpr (PAIR)
+            tc_commit_pair_multicast(&empty[stage], 0x3);
+          else
+            tc_commit(&empty[stage]);
           if (++stage == S) {
             stage = 0;
             phase ^= 1;
           }
         }
-        if (ok) tc_commit(&tfull[acc]);
+        if (ok) {
+          if constexpr (PAIR)
+            tc_commit_pair_multicast(&tfull[acc], 0x3);
+          else
+            tc_commit(&tfull[acc]);
+        }
       }
       if (!ok) record_status(args.status, ELASTO_ERR_TIMEOUT);
       // All MMAs this thread issued have finished once `drain` completes.
       if (issued) {
-        tc_commit(drain);
+        if constexpr (PAIR)
+          tc_commit_pair(drain);
+        else
+          tc_commit(drain);
         mbar_wait(drain, 0);
       }
     }
@@ -288,13 +342,13 @@ __global__ void __launch_bounds__(THREADS, 1)
     // the named barriers below can never be left one arrival short.
     volatile int* verdict = reinterpret_cast<volatile int*>(tmem_slot + 1);
     ChunkIter pf;  // residual prefetch iterator (elected thread only)
-    pf.init(tiles);
+    pf.init(tiles, t_start, t_stride);
     long loads = 0, consumed = 0, stored = 0;
     if constexpr (TR::resid) {
       if (elected) {
         for (int e = 0; e < E && pf.valid; ++e) {
           mbar_expect_tx(&rfull[e], CBUF);
-          tma_load_2d(sC + e * CBUF, &tmR, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
+          tma_load_2d(sC + e * CBUF, &tmR, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * TM + rank * BM);
           pf.advance(tiles, nt, bn, CW, N);
           ++loads;
         }
@@ -304,17 +358,18 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint32_t rph = 0;
     bool ok = true;
     int local = 0;
-    for (int t = blockIdx.x; t < tiles && ok; t += gridDim.x, ++local) {
+    for (int t = t_start; t < tiles && ok; t += t_stride, ++local) {
       const int acc = local & 1;
       const uint32_t use = static_cast<uint32_t>(local >> 1);
-      if (elected) *verdict = mbar_wait(&tfull[acc], use & 1) ? 1 : 0;
+      if (elected)
+        *verdict = (PAIR ? mbar_wait_cluster(&tfull[acc], use & 1) : mbar_wait(&tfull[acc], use & 1)) ? 1 : 0;
       named_bar_sync(1, EPI_THREADS);
       if (!*verdict) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const int m0 = (t / nt) * BM, n0 = (t % nt) * bn;
+      const int m0 = (t / nt) * TM + rank * BM, n0 = (t % nt) * bn;
       const uint32_t acc_tm = row_tm + acc * MAX_BN;
       int nvalid = 0;
       while (nvalid < cpt && n0 + nvalid * CW < N) ++nvalid;
@@ -348,7 +403,12 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           if (c == nvalid - 1) {  // last TMEM read of this tile
             tc_fence_before();
-            if (lane == 0) mbar_arrive(&tempty[acc]);
+            if (lane == 0) {
+              if constexpr (PAIR)
+                mbar_arrive_cluster(cluster_map(smem_addr(&tempty[acc]), 0));  // the even CTA issues the MMAs
+              else
+                mbar_arrive(&tempty[acc]);
+            }
           }
           float bb[HW];
           load_bias<HW>(args.bias, n0 + c * CW + g * HW, N, bb);
@@ -393,7 +453,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (stored > 0 && pf.valid) {
               const int ep = e == 0 ? E - 1 : e - 1;  // buffer of the previous chunk
               mbar_expect_tx(&rfull[ep], CBUF);
-              tma_load_2d(sC + ep * CBUF, &tmR, &rfull[ep], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * BM);
+              tma_load_2d(sC + ep * CBUF, &tmR, &rfull[ep], (pf.t % nt) * bn + pf.c * CW,
+                          (pf.t / nt) * TM + rank * BM);
               pf.advance(tiles, nt, bn, CW, N);
               ++loads;
             }
@@ -428,7 +489,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     float* st = reinterpret_cast<float*>(sC) + (warp - 2) * EPI_TILE;
     int local = 0;
-    for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++local) {
+    for (int t = t_start; t < tiles; t += t_stride, ++local) {
       const int acc = local & 1;
       const uint32_t use = static_cast<uint32_t>(local >> 1);
       if (!mbar_wait(&tfull[acc], use & 1)) {
@@ -436,7 +497,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       tc_fence_after();
-      const int m0 = (t / nt) * BM, n0 = (t % nt) * bn;
+      const int m0 = (t / nt) * TM + rank * BM, n0 = (t % nt) * bn;
       const int row0 = m0 + q * 32;
       for (int c = 0; c < bn; c += 32) {
         if (n0 + c >= N) break;
@@ -501,22 +562,56 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     }
   }
+  tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) cluster_sync_all();  // the peer's TMEM and barriers are no longer in use
   if (warp == 0) {
     __syncwarp();
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    if constexpr (PAIR)
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else
+      tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
-template <int EPI, int NB>
+template <int EPI, int NB, bool PAIR>
 cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   GemmArgs a = p.args;
   a.M = M;
-  const int tiles = ((M + BM - 1) / BM) * ((a.N + a.bn - 1) / a.bn);
-  const int grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_tc_kernel<EPI, NB><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
-  return cudaGetLastError();
+  const int nt = (a.N + a.bn - 1) / a.bn;
+  if constexpr (PAIR) {
+    static int max_clusters[64] = {0};
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaLaunchConfig_t cfg{};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = SMEM_BYTES;
+    cfg.stream = s;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (dev >= 0 && dev < 64 && max_clusters[dev] == 0) {
+      cfg.gridDim = dim3(2 * (num_sms() / 2));
+      int n = 0;
+      cudaError_t e = cudaOccupancyMaxActiveClusters(&n, gemm_tc_kernel<EPI, NB, true>, &cfg);
+      if (e != cudaSuccess || n <= 0) return e != cudaSuccess ? e : cudaErrorInvalidConfiguration;
+      max_clusters[dev] = n;
+    }
+    const int tiles = ((M + 2 * BM - 1) / (2 * BM)) * nt;
+    const int clusters = tiles < max_clusters[dev] ? tiles : max_clusters[dev];
+    cfg.gridDim = dim3(2 * clusters);
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<EPI, NB, true>, p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
+  } else {
+    const int tiles = ((M + BM - 1) / BM) * nt;
+    const int grid = tiles < num_sms() ? tiles : num_sms();
+    gemm_tc_kernel<EPI, NB, false><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
+    return cudaGetLastError();
+  }
 }
 
 }  // namespace
@@ -524,10 +619,13 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
 cudaError_t gemm_init_attributes() {
   const int bytes = static_cast<int>(SMEM_BYTES);
   cudaError_t e;
-#define SET_ATTR(E)                                                                                     \
-  e = cudaFuncSetAttribute(gemm_tc_kernel<E, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);   \
-  if (e != cudaSuccess) return e;                                                                       \
-  e = cudaFuncSetAttribute(gemm_tc_kernel<E, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);   \
+#define SET_ATTR(E)                                                                                        \
+  e = cudaFuncSetAttribute(gemm_tc_kernel<E, 1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);   \
+  if (e != cudaSuccess) return e;                                                                          \
+  e = cudaFuncSetAttribute(gemm_tc_kernel<E, 2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);   \
+  if (e != cudaSuccess) return e;
+#define SET_ATTR_PAIR(E)                                                                                   \
+  e = cudaFuncSetAttribute(gemm_tc_kernel<E, 1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);    \
   if (e != cudaSuccess) return e;
   SET_ATTR(EPI_BIAS_BF16)
   SET_ATTR(EPI_BIAS_GELU_BF16)
@@ -536,19 +634,25 @@ cudaError_t gemm_init_attributes() {
   SET_ATTR(EPI_BIAS_RELU_BF16)
   SET_ATTR(EPI_BIAS_RESID_RELU_BF16)
   SET_ATTR(EPI_PATCH_POS_F32)
+  SET_ATTR_PAIR(EPI_BIAS_BF16)
+  SET_ATTR_PAIR(EPI_BIAS_GELU_BF16)
+  SET_ATTR_PAIR(EPI_BIAS_RESID_F32)
+  SET_ATTR_PAIR(EPI_BIAS_RELU_BF16)
 #undef SET_ATTR
+#undef SET_ATTR_PAIR
   return cudaSuccess;
 }
 
-int gemm_pick_bn(int M, int N, int step) {
+int gemm_pick_bn(int M, int N, int step, bool pair) {
   // Estimated time ~ waves x (bn + fixed per-tile overhead); ties prefer wider tiles.
   const int sms = num_sms() > 0 ? num_sms() : 148;
-  const int mt = (M + BM - 1) / BM;
+  const int units = pair ? sms / 2 : sms;  // concurrent tile workers
+  const int mt = (M + (pair ? 2 * BM : BM) - 1) / (pair ? 2 * BM : BM);
   int best = 256;
   long best_cost = -1;
   for (int bn = 256; bn >= step; bn -= step) {
     const long tiles = static_cast<long>(mt) * ((N + bn - 1) / bn);
-    const long waves = (tiles + sms - 1) / sms;
+    const long waves = (tiles + units - 1) / units;
     const long cost = waves * (bn + 32);
     if (best_cost < 0 || cost < best_cost) {
       best_cost = cost;
@@ -576,8 +680,14 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   a.M = M_cap;
   a.N = N;
   a.K = K;
+  // CTA pairs for the TMA-store epilogues on problems with at least one
+  // 256-row tile and single-plane weights
+  // (long reductions only: with K = 768 the per-tile epilogue dominates and
+  // a single CTA per tile measured faster)
+  const bool pair = tma_out && !W_lo && M_cap >= 2 * BM && K >= 1536;
+  a.pair = pair ? 1 : 0;
   // bf16 staging chunks are 64 columns wide: their tiles are multiples of 64
-  a.bn = gemm_pick_bn(M_cap, N, (tma_out && !f32_out) ? 64 : 32);
+  a.bn = gemm_pick_bn(M_cap, N, (tma_out && !f32_out) ? 64 : 32, pair);
   a.bias = bias;
   a.out = out;
   a.ldo = ldo;
@@ -587,8 +697,13 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   if (tma_out) {
     // residual GEMMs: 3 operand stages and 5 staging chunks fetched ahead;
     // the others: 4 stages and 2 staging chunks.
-    a.stages = W_lo ? 2 : (f32_out ? 3 : 4);
-    a.cbufs = (POOL - a.stages * (A_STAGE + a.b_planes * B_STAGE)) / CBUF;
+    if (pair) {
+      a.stages = f32_out ? 5 : 6;
+      a.cbufs = (POOL - a.stages * (A_STAGE + B_STAGE_PAIR)) / CBUF;
+    } else {
+      a.stages = W_lo ? 2 : (f32_out ? 3 : 4);
+      a.cbufs = (POOL - a.stages * (A_STAGE + a.b_planes * B_STAGE)) / CBUF;
+    }
     if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
     if (ldo % 8 != 0 ||
         !encode_tmap_2d(&p->tmC, out, ldo, M_cap, static_cast<uint64_t>(ldo) * (f32_out ? 4 : 2),
@@ -598,12 +713,22 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     }
     p->tmR = p->tmC;  // the residual is read from the output unless redirected
   } else {
-    a.stages = W_lo ? 2 : MAX_STAGES;
+    a.stages = W_lo ? 2 : 4;
     a.cbufs = 0;
+  }
+  {
+    // the operand ring, staging chunks (or transpose tiles) must fit the pool
+    const int bstg = pair ? B_STAGE_PAIR : a.b_planes * B_STAGE;
+    const int tail = tma_out ? a.cbufs * CBUF : 4 * EPI_TILE * 4;
+    if (a.stages < 2 || a.stages > MAX_STAGES || a.cbufs > MAX_CBUFS || (tma_out && a.cbufs < 2) ||
+        a.stages * (A_STAGE + bstg) + tail > POOL) {
+      set_error("gemm_plan: shared-memory layout does not fit");
+      return ELASTO_ERR_UNSUPPORTED;
+    }
   }
   if (K > 0) {
     if (!encode_tmap_2d(&p->tmA, A, K, M_cap, static_cast<uint64_t>(K) * 2, BK, BM) ||
-        !encode_tmap_2d(&p->tmB, W, K, N, static_cast<uint64_t>(K) * 2, BK, a.bn) ||
+        !encode_tmap_2d(&p->tmB, W, K, N, static_cast<uint64_t>(K) * 2, BK, pair ? a.bn / 2 : a.bn) ||
         (W_lo && !encode_tmap_2d(&p->tmB2, W_lo, K, N, static_cast<uint64_t>(K) * 2, BK, a.bn))) {
       set_error("gemm_plan: cuTensorMapEncodeTiled failed (alignment or size)");
       return ELASTO_ERR_UNSUPPORTED;
@@ -628,18 +753,23 @@ elasto_status gemm_set_residual_source(GemmPlan* p, const float* src, int M_cap)
 
 cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s) {
   if (M <= 0) return cudaSuccess;
-  const bool two = p.args.b_planes == 2;
+  const bool two = p.args.b_planes == 2, pair = p.args.pair != 0;
 #define CASE(E) \
-  case E: return two ? launch_epi<E, 2>(p, M, s) : launch_epi<E, 1>(p, M, s);
+  case E: return two ? launch_epi<E, 2, false>(p, M, s) : launch_epi<E, 1, false>(p, M, s);
+#define CASE_PAIR(E)                                   \
+  case E:                                              \
+    if (pair) return launch_epi<E, 1, true>(p, M, s);  \
+    return two ? launch_epi<E, 2, false>(p, M, s) : launch_epi<E, 1, false>(p, M, s);
   switch (p.epi) {
-    CASE(EPI_BIAS_BF16)
-    CASE(EPI_BIAS_GELU_BF16)
-    CASE(EPI_BIAS_RESID_F32)
+    CASE_PAIR(EPI_BIAS_BF16)
+    CASE_PAIR(EPI_BIAS_GELU_BF16)
+    CASE_PAIR(EPI_BIAS_RESID_F32)
     CASE(EPI_BIAS_F32)
-    CASE(EPI_BIAS_RELU_BF16)
+    CASE_PAIR(EPI_BIAS_RELU_BF16)
     CASE(EPI_BIAS_RESID_RELU_BF16)
     CASE(EPI_PATCH_POS_F32)
 #undef CASE
+#undef CASE_PAIR
     default: return cudaErrorInvalidValue;
   }
 }
