@@ -54,9 +54,10 @@ enum { ELASTO_F32 = 0, ELASTO_BF16 = 1 };
  * ResNet-50 v1.5: img_c = 3, classes C; patch/dim/heads/mlp/layers ignored
  *   (bottlenecks [3,4,6,3], widths 64..512 are fixed).
  * weight_dtype: storage type of the weights AND of the images given to
- *   forward (ELASTO_F32 or ELASTO_BF16). Weights are stored on the device as
- *   bf16 (fp32 inputs are rounded to nearest even); biases, LayerNorm
- *   parameters, position embeddings and the classifier stay fp32.
+ *   forward (ELASTO_F32 or ELASTO_BF16). ViT weights are stored on the device
+ *   as bf16 (fp32 inputs as a bf16 hi + lo pair); ResNet-50 convolution
+ *   weights (BN folded) and activations as IEEE f16; biases, LayerNorm
+ *   parameters, position embeddings and the classifiers stay fp32.
  * max_batch: largest batch forward accepts; sizes the activation workspace. */
 typedef struct {
   int arch;
@@ -208,8 +209,9 @@ elasto_status elasto_profile_read(elasto_t h, elasto_launch_record* out, int cap
  * equal its size). ViT `which`: 0 qkv_w bf16 [3w,d], 1 qkv_b fp32 [3w],
  * 2 proj_w bf16 [d,w], 3 fc1_w bf16 [f,d], 4 fc1_b fp32 [f], 5 fc2_w bf16 [d,f]
  * (w = 64 x kept heads, f = kept channels). ResNet-50 (layer = block):
- * 0 conv1 bf16 [|S_a|, cin], 1 bias1 fp32, 2 conv2 bf16 [|S_b|, 3, 3, |S_a|],
- * 3 bias2 fp32, 4 conv3 bf16 [4w, |S_b|], 5 bias3 fp32 (BN folded).
+ * 0 conv1 f16 [|S_a|, cin], 1 bias1 fp32, 2 conv2 f16 [|S_b|, 3, 3, |S_a|],
+ * 3 bias2 fp32, 4 conv3 f16 [4w, |S_b|], 5 bias3 fp32 (BN folded; the
+ * ResNet path computes with IEEE f16 operands and fp32 accumulation).
  * Synchronous. Errors: INVALID_ARG, BAD_MODE. */
 elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int which, void* host_dst,
                                          size_t bytes);

@@ -27,7 +27,12 @@ typedef enum {
   ELASTO_EPI_BIAS_RESID_F32 = 2,  /* out fp32 += acc + bias                 (proj, FC2: residual) */
   ELASTO_EPI_BIAS_F32 = 3,        /* out fp32 = acc + bias */
   ELASTO_EPI_BIAS_RELU_BF16 = 4,  /* out bf16 = ReLU(acc + bias)            (conv + folded BN) */
-  ELASTO_EPI_BIAS_RESID_RELU_BF16 = 5 /* out bf16 = ReLU(acc + bias + resid) (block output) */
+  ELASTO_EPI_BIAS_RESID_RELU_BF16 = 5, /* out bf16 = ReLU(acc + bias + resid) (block output) */
+  /* The same with A, W, resid and out in IEEE f16 (ResNet-50 path: f16 has
+   * 3 more mantissa bits than bf16 at the same tensor-core rate) */
+  ELASTO_EPI_BIAS_RELU_F16 = 6,       /* out f16 = ReLU(acc + bias)             (conv + folded BN) */
+  ELASTO_EPI_BIAS_F16 = 7,            /* out f16 = acc + bias                   (shortcut projection) */
+  ELASTO_EPI_BIAS_RESID_RELU_F16 = 8  /* out f16 = ReLU(acc + bias + resid)     (block output) */
 } elasto_epilogue;
 
 /* out[M,N] = epilogue(A[M,K] W[N,K]^T): A, W bf16 (K contiguous); bias fp32

@@ -24,6 +24,7 @@ OK, ERR_INVALID_ARG, ERR_BAD_TABLE, ERR_BAD_MODE, ERR_OOM, ERR_CUDA, ERR_UNSUPPO
     0, -1, -2, -3, -4, -5, -6, -7)
 Q_N_MODES, Q_PACKED_BYTES, Q_SHARED_BYTES, Q_WORKSPACE_BYTES, Q_ARENA_BYTES, Q_MODE_MACS, Q_LAUNCHES = range(7)
 EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_BIAS_RESID_F32, EPI_BIAS_F32, EPI_BIAS_RELU_BF16, EPI_BIAS_RESID_RELU_BF16 = range(6)
+EPI_BIAS_RELU_F16, EPI_BIAS_F16, EPI_BIAS_RESID_RELU_F16 = range(6, 9)  # A, W, resid, out in IEEE f16
 
 c_int, c_void_p, c_size_t, c_int64 = ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int64
 P_i32 = ctypes.POINTER(ctypes.c_int32)

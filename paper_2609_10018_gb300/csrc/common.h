@@ -2,6 +2,7 @@
 #pragma once
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -45,6 +46,9 @@ enum GemmEpi : int {
   EPI_BIAS_F32 = ELASTO_EPI_BIAS_F32,
   EPI_BIAS_RELU_BF16 = ELASTO_EPI_BIAS_RELU_BF16,
   EPI_BIAS_RESID_RELU_BF16 = ELASTO_EPI_BIAS_RESID_RELU_BF16,
+  EPI_BIAS_RELU_F16 = ELASTO_EPI_BIAS_RELU_F16,
+  EPI_BIAS_F16 = ELASTO_EPI_BIAS_F16,
+  EPI_BIAS_RESID_RELU_F16 = ELASTO_EPI_BIAS_RESID_RELU_F16,
   EPI_PATCH_POS_F32 = 16,  // patch embedding: out row remapped past the class token, + position embedding
 };
 
@@ -64,6 +68,7 @@ struct GemmArgs {
   int cbufs;              // output staging buffers (16 KB each) for the TMA-store epilogues
   int b_planes;           // 2: W held as bf16 hi + lo planes (fp32-stored models), both multiplied
   int pair;               // 1: clusters of two CTAs sharing 256-row tiles (tcgen05 cta_group::2)
+  int f16;                // 1: A, W, the residual and 16-bit outputs are f16 (the *_F16 epilogues), else bf16
 };
 
 struct GemmPlan {

@@ -69,8 +69,9 @@ __device__ __forceinline__ float gelu(float x) {
 
 template <int EPI>
 struct EpiTraits {
+  static constexpr bool half = EPI == EPI_BIAS_RELU_F16 || EPI == EPI_BIAS_F16 || EPI == EPI_BIAS_RESID_RELU_F16;
   static constexpr bool tma = EPI == EPI_BIAS_BF16 || EPI == EPI_BIAS_GELU_BF16 || EPI == EPI_BIAS_RELU_BF16 ||
-                              EPI == EPI_BIAS_RESID_F32;
+                              EPI == EPI_BIAS_RESID_F32 || EPI == EPI_BIAS_RELU_F16 || EPI == EPI_BIAS_F16;
   static constexpr bool f32 = EPI == EPI_BIAS_RESID_F32;
   static constexpr bool resid = EPI == EPI_BIAS_RESID_F32;
   static constexpr int cw = f32 ? 32 : 64;  // columns per 128-byte staging chunk
@@ -79,8 +80,17 @@ struct EpiTraits {
 template <int EPI>
 __device__ __forceinline__ float epi_act(float v) {
   if constexpr (EPI == EPI_BIAS_GELU_BF16) return gelu(v);
-  if constexpr (EPI == EPI_BIAS_RELU_BF16) return fmaxf(v, 0.0f);
+  if constexpr (EPI == EPI_BIAS_RELU_BF16 || EPI == EPI_BIAS_RELU_F16) return fmaxf(v, 0.0f);
   return v;
+}
+
+// Two fp32 values -> one 32-bit word of the epilogue's 16-bit output type.
+template <int EPI>
+__device__ __forceinline__ uint32_t pack_out(float lo, float hi) {
+  if constexpr (EpiTraits<EPI>::half)
+    return pack_f16x2(lo, hi);
+  else
+    return pack_bf16x2(lo, hi);
 }
 
 // W consecutive bias values starting at column col (zero past N or if null).
@@ -259,7 +269,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0 && leader) {
-      const uint32_t idesc = idesc_bf16_f32(TM, bn);
+      const uint32_t idesc = idesc_16_f32(TM, bn, args.f16 != 0);
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true, issued = false;
@@ -428,13 +438,13 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
             for (int j = 0; j < NC; ++j) {
               uint4 pk;
-              pk.x = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 0]) + bb[8 * j + 0]),
+              pk.x = pack_out<EPI>(epi_act<EPI>(__uint_as_float(v[8 * j + 0]) + bb[8 * j + 0]),
                                  epi_act<EPI>(__uint_as_float(v[8 * j + 1]) + bb[8 * j + 1]));
-              pk.y = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 2]) + bb[8 * j + 2]),
+              pk.y = pack_out<EPI>(epi_act<EPI>(__uint_as_float(v[8 * j + 2]) + bb[8 * j + 2]),
                                  epi_act<EPI>(__uint_as_float(v[8 * j + 3]) + bb[8 * j + 3]));
-              pk.z = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 4]) + bb[8 * j + 4]),
+              pk.z = pack_out<EPI>(epi_act<EPI>(__uint_as_float(v[8 * j + 4]) + bb[8 * j + 4]),
                                  epi_act<EPI>(__uint_as_float(v[8 * j + 5]) + bb[8 * j + 5]));
-              pk.w = pack_bf16x2(epi_act<EPI>(__uint_as_float(v[8 * j + 6]) + bb[8 * j + 6]),
+              pk.w = pack_out<EPI>(epi_act<EPI>(__uint_as_float(v[8 * j + 6]) + bb[8 * j + 6]),
                                  epi_act<EPI>(__uint_as_float(v[8 * j + 7]) + bb[8 * j + 7]));
               *reinterpret_cast<uint4*>(rowp + (((NC * g + j) ^ (r & 7)) << 4)) = pk;
             }
@@ -536,7 +546,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
           }
         } else {
-          // EPI_BIAS_RESID_RELU_BF16
+          // EPI_BIAS_RESID_RELU_BF16 / _F16
           const int cp = (lane & 15) * 2;
           const int col = n0 + c + cp;
           const bool cok = col < N;
@@ -548,11 +558,20 @@ __global__ void __launch_bounds__(THREADS, 1)
             const int rr = 2 * i + (lane >> 4);
             const int row = row0 + rr;
             if (!(cok && row < M)) continue;
-            const __nv_bfloat162 rv =
-                *reinterpret_cast<const __nv_bfloat162*>(args.resid + static_cast<size_t>(row) * args.ldr + col);
-            const float v0 = fmaxf(st[rr * EPI_LD + cp] + b0 + __bfloat162float(rv.x), 0.0f);
-            const float v1 = fmaxf(st[rr * EPI_LD + cp + 1] + b1 + __bfloat162float(rv.y), 0.0f);
-            out[(static_cast<size_t>(row) * args.ldo + col) >> 1] = pack_bf16x2(v0, v1);
+            const uint32_t rw =
+                *reinterpret_cast<const uint32_t*>(args.resid + static_cast<size_t>(row) * args.ldr + col);
+            float r0, r1;
+            if constexpr (TR::half) {
+              const float2 rf = __half22float2(*reinterpret_cast<const __half2*>(&rw));
+              r0 = rf.x;
+              r1 = rf.y;
+            } else {
+              r0 = __uint_as_float(rw << 16);
+              r1 = __uint_as_float(rw & 0xffff0000u);
+            }
+            const float v0 = fmaxf(st[rr * EPI_LD + cp] + b0 + r0, 0.0f);
+            const float v1 = fmaxf(st[rr * EPI_LD + cp + 1] + b1 + r1, 0.0f);
+            out[(static_cast<size_t>(row) * args.ldo + col) >> 1] = pack_out<EPI>(v0, v1);
           }
         }
         __syncwarp();
@@ -634,6 +653,11 @@ cudaError_t gemm_init_attributes() {
   SET_ATTR(EPI_BIAS_RELU_BF16)
   SET_ATTR(EPI_BIAS_RESID_RELU_BF16)
   SET_ATTR(EPI_PATCH_POS_F32)
+  SET_ATTR(EPI_BIAS_RELU_F16)
+  SET_ATTR(EPI_BIAS_F16)
+  SET_ATTR(EPI_BIAS_RESID_RELU_F16)
+  SET_ATTR_PAIR(EPI_BIAS_RELU_F16)
+  SET_ATTR_PAIR(EPI_BIAS_F16)
   SET_ATTR_PAIR(EPI_BIAS_BF16)
   SET_ATTR_PAIR(EPI_BIAS_GELU_BF16)
   SET_ATTR_PAIR(EPI_BIAS_RESID_F32)
@@ -674,9 +698,10 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   }
   *p = GemmPlan{};
   const bool tma_out = epi == EPI_BIAS_BF16 || epi == EPI_BIAS_GELU_BF16 || epi == EPI_BIAS_RELU_BF16 ||
-                       epi == EPI_BIAS_RESID_F32;
+                       epi == EPI_BIAS_RESID_F32 || epi == EPI_BIAS_RELU_F16 || epi == EPI_BIAS_F16;
   const bool f32_out = epi == EPI_BIAS_RESID_F32;
   GemmArgs& a = p->args;
+  a.f16 = (epi == EPI_BIAS_RELU_F16 || epi == EPI_BIAS_F16 || epi == EPI_BIAS_RESID_RELU_F16) ? 1 : 0;
   a.M = M_cap;
   a.N = N;
   a.K = K;
@@ -768,6 +793,9 @@ cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s) {
     CASE_PAIR(EPI_BIAS_RELU_BF16)
     CASE(EPI_BIAS_RESID_RELU_BF16)
     CASE(EPI_PATCH_POS_F32)
+    CASE_PAIR(EPI_BIAS_RELU_F16)
+    CASE_PAIR(EPI_BIAS_F16)
+    CASE(EPI_BIAS_RESID_RELU_F16)
 #undef CASE
 #undef CASE_PAIR
     default: return cudaErrorInvalidValue;

@@ -11,8 +11,8 @@ extern "C" {
 elasto_status elasto_op_gemm(void* stream, const void* A, const void* W, const float* bias, void* out,
                              const void* resid, int M, int N, int K, int epilogue, int* status_device) {
   clear_error();
-  if (!out || M <= 0 || N <= 0 || K < 0 || (K > 0 && (!A || !W)) || epilogue < 0 || epilogue > 5 ||
-      (epilogue == ELASTO_EPI_BIAS_RESID_RELU_BF16 && !resid)) {
+  if (!out || M <= 0 || N <= 0 || K < 0 || (K > 0 && (!A || !W)) || epilogue < 0 || epilogue > 8 ||
+      ((epilogue == ELASTO_EPI_BIAS_RESID_RELU_BF16 || epilogue == ELASTO_EPI_BIAS_RESID_RELU_F16) && !resid)) {
     set_error("elasto_op_gemm: invalid arguments");
     return ELASTO_ERR_INVALID_ARG;
   }

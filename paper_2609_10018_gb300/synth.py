@@ -245,7 +245,8 @@ def resnet_weight_shapes(cfg: ResnetConfig) -> Dict[str, Tuple[int, ...]]:
 
 
 def make_resnet_weights(cfg: ResnetConfig, seed: int | None = None) -> Dict[str, np.ndarray]:
-    """He-normal convs; BN gamma U(0.5, 1) (U(0.1, 0.3) on a block's last BN),
+    """He-normal convs; BN gamma U(0.5, 1) (U(0.1, 0.3) on bn3, the last BN of a
+    block's residual branch),
     beta N(0, 0.05), running mean N(0, 0.1), running var U(0.5, 1.5); FC N(0, 0.01)."""
     rng = np.random.default_rng(cfg.seeds[0] if seed is None else seed)
     shapes = resnet_weight_shapes(cfg)
@@ -258,7 +259,11 @@ def make_resnet_weights(cfg: ResnetConfig, seed: int | None = None) -> Dict[str,
         elif name == "fc_w" or name == "fc_b":
             x = rng.standard_normal(shp, dtype=np.float32) * np.float32(0.01)
         elif name.endswith(".g"):
-            lo, hi = (0.1, 0.3) if (".bn3." in name or ".down_bn." in name) else (0.5, 1.0)
+            # only the BN closing a block's residual branch is small (bounds the
+            # growth of the residual sum); the shortcut projection's BN is not,
+            # or four projections would shrink the image signal ~0.2^4 against
+            # the constant BN shifts and every image would get the same logits
+            lo, hi = (0.1, 0.3) if ".bn3." in name else (0.5, 1.0)
             x = rng.uniform(lo, hi, shp).astype(np.float32)
         elif name.endswith(".b"):
             x = rng.standard_normal(shp, dtype=np.float32) * np.float32(0.05)

@@ -99,3 +99,63 @@ def test_wrong_tensor_count_rejected(lib):
 
 def test_build_flags_target_sm103a_only():
     assert builder.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def _resnet_args(tables=None, **desc_kw):
+    import dataclasses
+    cfg = dataclasses.replace(synth.RESNET50, img=32, classes=10)
+    keep = binding._Keep()
+    w = synth.make_resnet_weights(cfg)
+    desc = binding.resnet_desc(cfg, 4)
+    for k, v in desc_kw.items():
+        setattr(desc, k, v)
+    tables = tables if tables is not None else synth.make_resnet_tables(cfg)
+    mt = binding.resnet_mode_tables(keep, tables)
+    ws = binding.weights_struct(keep, [w[k] for k in synth.resnet_weight_names(cfg)])
+    return keep, desc, ws, mt, len(tables)
+
+
+@pytest.mark.parametrize("mutate", [
+    lambda t: t[2]["a"].__setitem__(0, np.array([3, 1], np.int32)),            # unsorted
+    lambda t: t[2]["b"].__setitem__(5, np.array([0, 0], np.int32)),            # duplicate
+    lambda t: t[2]["a"].__setitem__(15, np.array([0, 512], np.int32)),         # out of range (width 512)
+    lambda t: t[2]["b"].__setitem__(1, np.zeros(0, np.int32)),                 # empty kept set
+    lambda t: t[2]["a"].__setitem__(0, np.arange(65, dtype=np.int32)),         # more than the width
+])
+def test_resnet_bad_tables_rejected_before_cuda(lib, mutate):
+    import dataclasses
+    tables = synth.make_resnet_tables(dataclasses.replace(synth.RESNET50, img=32, classes=10))
+    mutate(tables)
+    keep, desc, ws, mt, n = _resnet_args(tables)
+    assert _create(lib, desc, ws, mt, n) == binding.ERR_BAD_TABLE
+    assert "mode 2" in binding.elasto_last_error()
+
+
+@pytest.mark.parametrize("field, value", [("img_c", 4), ("img_h", 16), ("classes", 0)])
+def test_resnet_bad_descriptor_rejected(lib, field, value):
+    keep, desc, ws, mt, n = _resnet_args(**{field: value})
+    assert _create(lib, desc, ws, mt, n) == binding.ERR_INVALID_ARG
+
+
+def test_resnet_tensor_count_is_267(lib):
+    keep, desc, ws, mt, n = _resnet_args()
+    assert ws.n_tensors == 267
+    ws.n_tensors = 266
+    assert _create(lib, desc, ws, mt, n) == binding.ERR_INVALID_ARG
+    assert "267" in binding.elasto_last_error()
+
+
+def test_oracle_pool_matches_direct_call():
+    """The spawn pool used by the ResNet parity tests returns the oracle's own
+    logits (two 32x32 images, one per worker)."""
+    import dataclasses
+    from oracle import resnet as orr
+    from oracle.vit import widen_all
+    from oracle_pool import resnet_logits
+    cfg = dataclasses.replace(synth.RESNET50, img=32, classes=10)
+    tables = synth.make_resnet_tables(cfg)
+    img = synth.make_images(cfg, 2)
+    got = resnet_logits(cfg, tables, 1, img, chunk=1)
+    ref = orr.resnet_forward_sliced(widen_all(synth.make_resnet_weights(cfg)), cfg, tables[1]["a"], tables[1]["b"], img)
+    # equal up to the BLAS summation order (one thread per worker here)
+    assert np.max(np.abs(got - ref)) <= 1e-12 * np.max(np.abs(ref))

@@ -32,17 +32,36 @@ GEMM_CASES = [
     (130, 200, 136, binding.EPI_BIAS_RELU_BF16),      # conv-like K
     (130, 64, 72, binding.EPI_BIAS_RESID_RELU_BF16),
     (64, 1152, 384, binding.EPI_BIAS_GELU_BF16),      # ViT-S 75 % MLP, M below one tile
+    # f16 operands (ResNet-50 path)
+    (200, 48, 576, binding.EPI_BIAS_RELU_F16),        # 3x3 conv of 64 kept channels into 48
+    (130, 16, 72, binding.EPI_BIAS_F16),              # N below one 64-column chunk
+    (1537, 256, 2048, binding.EPI_BIAS_RELU_F16),     # K >= 1536: CTA-pair kernel with f16
+    (333, 1024, 136, binding.EPI_BIAS_RESID_RELU_F16),
+    (6272, 2048, 512, binding.EPI_BIAS_RESID_RELU_F16),  # last conv3 of ResNet-50 at batch 128
 ]
+
+F16_EPIS = (binding.EPI_BIAS_RELU_F16, binding.EPI_BIAS_F16, binding.EPI_BIAS_RESID_RELU_F16)
+
+
+def _f16(rng, shape, scale=1.0):
+    return (rng.standard_normal(shape, dtype=np.float32) * np.float32(scale)).astype(np.float16).view(np.uint16)
+
+
+def _f16_to_f64(bits):
+    a = bits.cpu().numpy() if hasattr(bits, "cpu") else np.asarray(bits)
+    return a.view(np.float16).astype(np.float64)
 
 
 @pytest.mark.parametrize("M,N,K,epi", GEMM_CASES)
 def test_gemm_epilogues_match_fp64(M, N, K, epi):
     import torch
     rng = np.random.default_rng(M * 7 + N * 3 + K)
-    A = _bf16(rng, (M, max(K, 8)))[:, :K].copy() if K else np.zeros((M, 0), np.uint16)
-    W = _bf16(rng, (N, max(K, 8)), 0.05)[:, :K].copy() if K else np.zeros((N, 0), np.uint16)
+    half = epi in F16_EPIS
+    gen, dec = (_f16, _f16_to_f64) if half else (_bf16, bf16_to_f64)
+    A = gen(rng, (M, max(K, 8)))[:, :K].copy() if K else np.zeros((M, 0), np.uint16)
+    W = gen(rng, (N, max(K, 8)), 0.05)[:, :K].copy() if K else np.zeros((N, 0), np.uint16)
     bias = rng.standard_normal(N).astype(np.float32)
-    ref = bf16_to_f64(A) @ bf16_to_f64(W).T + bias
+    ref = dec(A) @ dec(W).T + bias
     f32_out = epi in (binding.EPI_BIAS_F32, binding.EPI_BIAS_RESID_F32)
     resid = None
     if epi == binding.EPI_BIAS_RESID_F32:
@@ -55,10 +74,12 @@ def test_gemm_epilogues_match_fp64(M, N, K, epi):
         ref = ov.gelu(ref)
     elif epi == binding.EPI_BIAS_RELU_BF16:
         ref = np.maximum(ref, 0)
-    elif epi == binding.EPI_BIAS_RESID_RELU_BF16:
-        r = _bf16(rng, (M, N))
+    elif epi == binding.EPI_BIAS_RELU_F16:
+        ref = np.maximum(ref, 0)
+    elif epi in (binding.EPI_BIAS_RESID_RELU_BF16, binding.EPI_BIAS_RESID_RELU_F16):
+        r = gen(rng, (M, N))
         resid = dev(r)
-        ref = np.maximum(ref + bf16_to_f64(r), 0)
+        ref = np.maximum(ref + dec(r), 0)
     st = _status()
     dA = dev(A) if K else None
     dW = dev(W) if K else None
@@ -68,10 +89,12 @@ def test_gemm_epilogues_match_fp64(M, N, K, epi):
                            M, N, K, epi, st.data_ptr())
     torch.cuda.synchronize()
     assert int(st.item()) == 0
-    got = out.cpu().numpy().astype(np.float64) if f32_out else bf16_to_f64(out)
+    got = out.cpu().numpy().astype(np.float64) if f32_out else dec(out)
     scale = float(np.max(np.abs(ref)))
     if f32_out:
         assert np.all(np.abs(got - ref) <= 1e-5 * scale + 1e-6 * np.abs(ref)), float(np.max(np.abs(got - ref)))
+    elif half:  # one f16 rounding of the fp32 result
+        assert np.all(np.abs(got - ref) <= 2.0 ** -11 * np.abs(ref) + 1e-5 * scale), float(np.max(np.abs(got - ref)))
     else:  # one bf16 rounding of the fp32 result
         assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5 * scale), float(np.max(np.abs(got - ref)))
 
