@@ -47,6 +47,8 @@ def parse_args():
     p.add_argument("--batch", type=int, default=256)
     p.add_argument("--mode", type=int, default=0)
     p.add_argument("--quick", action="store_true", help="headline only: skip per-mode sweep, latency, e2e, baseline")
+    p.add_argument("--resnet-only", action="store_true",
+                   help="print only the ResNet-50 section (per-mode images/s at batch 128)")
     return p.parse_args()
 
 
@@ -226,6 +228,9 @@ def main():
 
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
+    if args.resnet_only:
+        print(json.dumps(resnet50_section(torch, binding, synth, load_peaks()[0])))
+        return
     dist = None
     if world > 1:
         import torch.distributed as dist
@@ -345,10 +350,71 @@ def main():
         line["e2e"] = e2e(model, cfg, images_np, B, args, torch, binding)
         line["cpu_baseline"] = oracle_cpu_baseline(cfg)
     model.close()
+    if rank == 0 and not args.quick:
+        line["resnet50"] = resnet50_section(torch, binding, synth, peaks)
     if rank == 0:
         print(json.dumps(line))
     if dist:
         dist.destroy_process_group()
+
+
+def resnet50_section(torch, binding, synth, peaks, B=128, steps=20, warmup=3):
+    """ResNet-50 DNs (Eq. 7) at 224x224, batch 128, every mode: images/s and
+    % of the dense 16-bit tensor peak (f16 operands run at the bf16 rate),
+    plus where mode 0's time goes, from the per-launch CUDA events."""
+    cfg = synth.RESNET50
+    w, tables = synth.make_resnet_weights(cfg), synth.make_resnet_tables(cfg)
+    model = binding.ElasticModel.resnet(cfg, w, tables, max_batch=B)
+    images = torch.from_numpy(synth.make_images(cfg, B)).cuda()
+    logits = torch.empty(B, cfg.classes, dtype=torch.float32, device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    out = {"workload": f"ResNet-50 v1.5 DN forward, 224x224, batch {B}, f16 operands / fp32 accumulation",
+           "l2": "flushed between timed steps", "per_mode": []}
+    for m in range(len(tables)):
+        model.set_mode(m)
+        for _ in range(warmup):
+            model.forward(sh, images.data_ptr(), B, logits.data_ptr())
+        torch.cuda.synchronize()
+        ts = []
+        for _ in range(steps):
+            flush.fill_(1.0)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            model.forward(sh, images.data_ptr(), B, logits.data_ptr())
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        ips = B * steps / (sum(ts) / 1e3)
+        macs = model.query(binding.Q_MODE_MACS, m)
+        tf = 2.0 * macs * ips / 1e12
+        out["per_mode"].append({"mode": m, "inner_width_frac": cfg.mode_frac[m], "images_per_s": ips,
+                                "ms_per_step": statistics.mean(ts), "tflops": tf,
+                                "frac_of_bf16_peak": tf / peaks["bf16_tflops"], "gflop_per_image": 2 * macs / 1e9,
+                                "packed_weight_mb": model.query(binding.Q_PACKED_BYTES, m) / 1e6,
+                                "launches": model.query(binding.Q_LAUNCHES, m)})
+    model.set_mode(0)
+    model.profile(True)
+    model.forward(sh, images.data_ptr(), B, logits.data_ptr())
+    recs = model.profile_read()
+    model.profile(False)
+    kinds = {}
+    for r in recs:
+        k = kinds.setdefault(r["kind"], {"ms": 0.0, "launches": 0, "macs": 0.0, "bytes": 0.0})
+        k["ms"] += r["ms"]
+        k["launches"] += 1
+        k["macs"] += r["macs"]
+        k["bytes"] += r["bytes"]
+    tot = sum(k["ms"] for k in kinds.values())
+    for k in kinds.values():
+        k["share"] = k["ms"] / tot
+        if k["macs"] > 0:
+            k["tflops"] = 2 * k["macs"] / (k["ms"] / 1e3) / 1e12
+        k["gbs"] = k["bytes"] / (k["ms"] / 1e3) / 1e9
+    out["mode0_kernels"] = kinds
+    model.close()
+    return out
 
 
 def batch1_latency(model, cfg, tables, torch, binding, peaks):

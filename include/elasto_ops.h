@@ -35,8 +35,9 @@ typedef enum {
   ELASTO_EPI_BIAS_RESID_RELU_F16 = 8  /* out f16 = ReLU(acc + bias + resid)     (block output) */
 } elasto_epilogue;
 
-/* out[M,N] = epilogue(A[M,K] W[N,K]^T): A, W bf16 (K contiguous); bias fp32
- * [N] or NULL (= 0); resid bf16 [M,N] only for ..._RESID_RELU_BF16. Output
+/* out[M,N] = epilogue(A[M,K] W[N,K]^T): A, W bf16 (f16 for the *_F16
+ * epilogues), K contiguous; bias fp32 [N] or NULL (= 0); resid [M,N] of the
+ * same 16-bit type only for the ..._RESID_RELU epilogues. Output
  * row stride is N. Requires K % 8 == 0, N % 2 == 0, M, N, K >= 1 (K may be 0:
  * then acc = 0). tcgen05 MMA (M = 128 tiles), TMA-fed, persistent grid. */
 elasto_status elasto_op_gemm(void* stream, const void* A, const void* W, const float* bias, void* out,
@@ -51,6 +52,19 @@ elasto_status elasto_op_layernorm(void* stream, const float* x, const float* gam
 /* y fp32 [rows, cols] = softmax over each row of x fp32 [rows, cols]
  * (exp(x - max) / sum, one warp per row, warp-shuffle reductions). */
 elasto_status elasto_op_softmax(void* stream, const float* x, float* y, int rows, int cols);
+
+/* k x k convolution (Eq. 7's conv over the kept channels) as an implicit
+ * GEMM: out f16 [B, Ho, Wo, N] = act(conv(x) + bias), Ho = (H + 2 pad - k) /
+ * stride + 1 (likewise Wo), act = ReLU if relu != 0 else identity.
+ *   x f16 [B, H, W, C] NHWC, C % 8 == 0;
+ *   w f16 [N, k, k, Cp] with Cp = C rounded up to 64, channels >= C zero
+ *     (the packed layout the ResNet path uses: one 64-channel group per
+ *     k-block of the tensor-core GEMM);
+ *   bias fp32 [N] or NULL. N % 2 == 0, stride 1 or 2.
+ * No im2col buffer: each k-block is one 4-D TMA tile of x (padding read as
+ * zeros, the stride by TMA traversal strides). */
+elasto_status elasto_op_conv2d(void* stream, const void* x, int B, int H, int W, int C, const void* w, int N, int k,
+                               int stride, int pad, const float* bias, int relu, void* out, int* status_device);
 
 /* Multi-head attention over the kept heads (Eq. 3), all heads of width 64:
  * qkv bf16 [batch, n, 3, heads, 64] (q | k | v blocks, head-major, as the

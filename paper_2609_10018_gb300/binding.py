@@ -88,6 +88,8 @@ def lib() -> ctypes.CDLL:
         "elasto_profile_read": [c_void_p, ctypes.POINTER(LaunchRecord), c_int, ctypes.POINTER(c_int)],
         "elasto_op_gemm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
                            c_void_p],
+        "elasto_op_conv2d": [c_void_p, c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int, c_int, c_int,
+                             c_void_p, c_int, c_void_p, c_void_p],
         "elasto_op_layernorm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int],
         "elasto_op_softmax": [c_void_p, c_void_p, c_void_p, c_int, c_int],
         "elasto_op_attention": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p],
@@ -250,6 +252,11 @@ def elasto_profile_read(h: int, capacity: int = 1024) -> List[dict]:
 
 def elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status=0) -> None:
     _check(lib().elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status), "elasto_op_gemm")
+
+
+def elasto_op_conv2d(stream, x, B, H, W, C, w, N, k, stride, pad, bias, relu, out, status=0) -> None:
+    _check(lib().elasto_op_conv2d(stream, x, B, H, W, C, w, N, k, stride, pad, bias, int(relu), out, status),
+           "elasto_op_conv2d")
 
 
 def elasto_op_layernorm(stream, x, gamma, beta, y, rows, d) -> None:

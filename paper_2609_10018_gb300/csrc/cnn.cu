@@ -14,10 +14,12 @@
 //   stem     7x7/2 conv: gather (ky, kx, c) patch rows, GEMM + bias + ReLU,
 //            then 3x3/2 max pool (padding never wins);
 //   block    conv1 1x1: GEMM straight on the NHWC activation [B*H*W, cin];
-//            conv2 3x3/stride: gather the 9 taps of the kept S_a channels
-//            ((ky, kx, c) columns), GEMM + bias + ReLU;
+//            conv2 3x3/stride: implicit GEMM (gemm_plan_conv): each k-block
+//            (tap, 64 kept channels) is a 4-D TMA tile of the conv1 output,
+//            padding read as zeros, stride by TMA traversal strides; + bias
+//            + ReLU;
 //            projection (first block of a stage): 1x1/stride conv + bias
-//            (a strided gather first when stride is 2);
+//            (an implicit GEMM too when the stride is 2);
 //            conv3 1x1: GEMM + bias + shortcut + ReLU in the epilogue;
 //   head     global average pool (fp32), classifier in fp32.
 //
@@ -62,6 +64,7 @@ using F16Buf = bf16;
 
 struct CnnBlockPack {
   int a = 0, b = 0, a_pad = 0, b_pad = 0;  // kept |S_a|, |S_b| and their padded widths
+  int a_cp = 0;                            // conv2's per-tap K stride: a_pad rounded up to 64
   F16Buf *w1 = nullptr, *w2 = nullptr, *w3 = nullptr;
   float *b1 = nullptr, *b2 = nullptr, *b3 = nullptr;
   GemmPlan conv1, conv2, conv3;
@@ -132,52 +135,42 @@ int n_tensors_expected() {
 
 // ---------------------------------------------------------------- kernels
 
-// dst[row, k] for k = (ky * kw + kx) * C + c of output pixel row = (b, oy, ox):
-// src[b, oy * stride - pad + ky, ox * stride - pad + kx, c], zero outside the
-// image and for k >= K (padding columns up to Kp).
+// The stem's gather (7x7, stride 2, padding 3, 3 channels, 152 columns with
+// 5 zero columns): one warp per output pixel, lane l writing columns l, l+32,
+// ..., so each warp store covers 64 contiguous bytes. A lane's (ky, kx, c)
+// are fixed for the whole kernel and computed once.
 template <typename T>
-__global__ void im2col_kernel(const T* __restrict__ src, int H, int W, int C, int kw, int stride, int pad, int Ho,
-                              int Wo, int K, int Kp, size_t total, __half* __restrict__ dst) {
-  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
-       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
-    const size_t row = t / Kp;
-    const int k = static_cast<int>(t - row * Kp);
-    float v = 0.0f;
-    if (k < K) {
-      const int tap = k / C, c = k - tap * C;
-      const int ky = tap / kw, kx = tap - ky * kw;
-      const int ox = static_cast<int>(row % Wo);
-      const size_t r2 = row / Wo;
-      const int oy = static_cast<int>(r2 % Ho);
-      const size_t b = r2 / Ho;
-      const int iy = oy * stride - pad + ky, ix = ox * stride - pad + kx;
-      if (iy >= 0 && iy < H && ix >= 0 && ix < W) {
-        v = static_cast<float>(src[((b * H + iy) * W + ix) * C + c]);
-      }
-    }
-    dst[t] = __float2half_rn(v);
+__global__ void __launch_bounds__(256) stem_im2col_kernel(const T* __restrict__ src, int H, int W, int Ho, int Wo,
+                                                          size_t rows, __half* __restrict__ dst) {
+  constexpr int NK = (kStemKp + 31) / 32;
+  const int lane = threadIdx.x & 31;
+  int dy[NK], dx[NK], dc[NK];
+#pragma unroll
+  for (int i = 0; i < NK; ++i) {
+    const int k = lane + 32 * i;
+    const int tap = k / 3;
+    dc[i] = k - 3 * tap;
+    dy[i] = k < kStemK ? tap / 7 : -1000;  // padding columns read nothing
+    dx[i] = tap - 7 * (tap / 7);
   }
-}
-
-// The same gather 16 bytes (8 channels) at a time: f16 source, C % 8 == 0,
-// no padding columns. Item t = ((row * taps) + tap) * C8 + c8.
-__global__ void im2col_vec_kernel(const uint4* __restrict__ src, int H, int W, int C8, int kw, int taps, int stride,
-                                  int pad, int Ho, int Wo, size_t total, uint4* __restrict__ dst) {
-  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
-       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
-    const int c8 = static_cast<int>(t % C8);
-    const size_t rest = t / C8;
-    const int tap = static_cast<int>(rest % taps);
-    const size_t row = rest / taps;
-    const int ky = tap / kw, kx = tap - ky * kw;
+  const size_t warps = static_cast<size_t>(gridDim.x) * (blockDim.x >> 5);
+  for (size_t row = static_cast<size_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); row < rows;
+       row += warps) {
     const int ox = static_cast<int>(row % Wo);
     const size_t r2 = row / Wo;
     const int oy = static_cast<int>(r2 % Ho);
     const size_t b = r2 / Ho;
-    const int iy = oy * stride - pad + ky, ix = ox * stride - pad + kx;
-    uint4 v = make_uint4(0u, 0u, 0u, 0u);
-    if (iy >= 0 && iy < H && ix >= 0 && ix < W) v = src[((b * H + iy) * W + ix) * C8 + c8];
-    dst[t] = v;
+    const T* img = src + b * H * W * 3;
+    __half* out = dst + row * kStemKp;
+#pragma unroll
+    for (int i = 0; i < NK; ++i) {
+      const int k = lane + 32 * i;
+      if (k >= kStemKp) break;
+      const int iy = 2 * oy - 3 + dy[i], ix = 2 * ox - 3 + dx[i];
+      float v = 0.0f;
+      if (iy >= 0 && iy < H && ix >= 0 && ix < W) v = static_cast<float>(img[(static_cast<size_t>(iy) * W + ix) * 3 + dc[i]]);
+      out[k] = __float2half_rn(v);
+    }
   }
 }
 
@@ -295,29 +288,17 @@ unsigned grid_for(size_t n) {
   return static_cast<unsigned>(b < 16384 ? (b > 0 ? b : 1) : 16384);
 }
 
-constexpr int kSrcF16 = 2;  // activations (besides ELASTO_F32 / ELASTO_BF16 images)
-
-// Gather for a k x k / stride / pad convolution of src [B, H, W, C] into
-// dst [B * Ho * Wo, Kp] f16.
-cudaError_t im2col_launch(const void* src, int src_dtype, int B, int H, int W, int C, int k, int stride, int pad,
-                          int Ho, int Wo, int Kp, __half* dst, cudaStream_t s) {
-  const int K = k * k * C;
+cudaError_t stem_im2col_launch(const void* images, int dtype, int B, int H, int W, int Ho, int Wo, __half* dst,
+                               cudaStream_t s) {
   const size_t rows = static_cast<size_t>(B) * Ho * Wo;
   if (rows == 0) return cudaSuccess;
-  if (src_dtype == kSrcF16 && C % 8 == 0 && Kp == K) {
-    const size_t total = rows * k * k * (C / 8);
-    im2col_vec_kernel<<<grid_for(total), 256, 0, s>>>(static_cast<const uint4*>(src), H, W, C / 8, k, k * k, stride,
-                                                      pad, Ho, Wo, total, reinterpret_cast<uint4*>(dst));
-  } else if (src_dtype == kSrcF16) {
-    im2col_kernel<__half><<<grid_for(rows * Kp), 256, 0, s>>>(static_cast<const __half*>(src), H, W, C, k, stride,
-                                                               pad, Ho, Wo, K, Kp, rows * Kp, dst);
-  } else if (src_dtype == ELASTO_BF16) {
-    im2col_kernel<bf16><<<grid_for(rows * Kp), 256, 0, s>>>(static_cast<const bf16*>(src), H, W, C, k, stride, pad,
-                                                             Ho, Wo, K, Kp, rows * Kp, dst);
-  } else {
-    im2col_kernel<float><<<grid_for(rows * Kp), 256, 0, s>>>(static_cast<const float*>(src), H, W, C, k, stride,
-                                                              pad, Ho, Wo, K, Kp, rows * Kp, dst);
-  }
+  const size_t blocks = std::min<size_t>((rows + 7) / 8, 16384);
+  if (dtype == ELASTO_BF16)
+    stem_im2col_kernel<bf16><<<unsigned(blocks), 256, 0, s>>>(static_cast<const bf16*>(images), H, W, Ho, Wo, rows,
+                                                              dst);
+  else
+    stem_im2col_kernel<float><<<unsigned(blocks), 256, 0, s>>>(static_cast<const float*>(images), H, W, Ho, Wo,
+                                                               rows, dst);
   return cudaGetLastError();
 }
 
@@ -485,10 +466,11 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
         bp.b = tables[mo].n_conv_b[i];
         bp.a_pad = round8(bp.a);
         bp.b_pad = round8(bp.b);
+        bp.a_cp = (bp.a_pad + 63) / 64 * 64;
         Off& o = offs[mo][i];
         o.w1 = ar.take(size_t(bp.a_pad) * S[i].cin * 2);
         o.b1 = ar.take(size_t(bp.a_pad) * 4);
-        o.w2 = ar.take(size_t(bp.b_pad) * 9 * bp.a_pad * 2);
+        o.w2 = ar.take(size_t(bp.b_pad) * 9 * bp.a_cp * 2);
         o.b2 = ar.take(size_t(bp.b_pad) * 4);
         o.w3 = ar.take(size_t(4) * S[i].w * bp.b_pad * 2);
         o.b3 = ar.take(size_t(4) * S[i].w * 4);
@@ -498,12 +480,11 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
   }
   // workspace (sizes for the widest mode: kept counts never exceed the width)
   const size_t rows_stem = size_t(Bm) * m->h1 * m->w1;
-  size_t col = rows_stem * kStemKp, xbuf = std::max(rows_stem * kStemC, size_t(Bm) * m->hp * m->wp * kStemC);
+  const size_t col = rows_stem * kStemKp;  // only the stem is gathered
+  size_t xbuf = std::max(rows_stem * kStemC, size_t(Bm) * m->hp * m->wp * kStemC);
   size_t t1 = 0, t2 = 0, scb = 0;
   for (const BlockShape& b : S) {
     const size_t ri = size_t(Bm) * b.hin * b.win, ro = size_t(Bm) * b.ho * b.wo;
-    col = std::max(col, ro * 9 * size_t(round8(b.w)));
-    if (b.proj && b.stride != 1) col = std::max(col, ro * size_t(b.cin));
     xbuf = std::max(xbuf, ro * 4 * size_t(b.w));
     t1 = std::max(t1, ri * size_t(round8(b.w)));
     t2 = std::max(t2, ro * size_t(round8(b.w)));
@@ -631,8 +612,8 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
       }
       ELASTO_CUDA_TRY(up16(bp.w1));
       ELASTO_CUDA_TRY(up32(bp.b1));
-      // conv2: rows S_b, input channels S_a, [b_pad, (ky, kx, c < a_pad)]
-      const size_t k2 = size_t(9) * bp.a_pad;
+      // conv2: rows S_b, input channels S_a, [b_pad, (ky, kx, c < a_cp)]
+      const size_t k2 = size_t(9) * bp.a_cp;
       hw.assign(size_t(bp.b_pad) * k2, 0);
       hb.assign(bp.b_pad, 0.0f);
       for (int r = 0; r < bp.b; ++r) {
@@ -641,7 +622,7 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
         for (int ky = 0; ky < 3; ++ky)
           for (int kx = 0; kx < 3; ++kx)
             for (int c = 0; c < bp.a; ++c)
-              hw[size_t(r) * k2 + size_t(ky * 3 + kx) * bp.a_pad + c] =
+              hw[size_t(r) * k2 + size_t(ky * 3 + kx) * bp.a_cp + c] =
                   f16_bits(static_cast<float>(W2[((size_t(o) * w + Sa[c]) * 3 + ky) * 3 + kx] * s));
         hb[r] = static_cast<float>(bn2.bias(o));
       }
@@ -672,8 +653,12 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
     F16Buf* xin = (i % 2 == 0) ? m->xa : m->xb;
     const int mo_cap = Bm * b.ho * b.wo;
     if (b.proj) {
-      st = gemm_plan(&m->down[i], b.stride == 1 ? xin : m->col, mo_cap, m->down_w[i], 4 * b.w, b.cin,
-                        m->down_b[i], m->sc, 4 * b.w, EPI_BIAS_F16, m->status);
+      if (b.stride == 1)
+        st = gemm_plan(&m->down[i], xin, mo_cap, m->down_w[i], 4 * b.w, b.cin, m->down_b[i], m->sc, 4 * b.w,
+                       EPI_BIAS_F16, m->status);
+      else
+        st = gemm_plan_conv(&m->down[i], xin, Bm, b.hin, b.win, b.cin, 1, b.stride, 0, m->down_w[i], 4 * b.w,
+                            m->down_b[i], m->sc, 4 * b.w, EPI_BIAS_F16, m->status);
       if (st != ELASTO_OK) return st;
     }
   }
@@ -690,17 +675,17 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
       st = gemm_plan(&bp.conv1, xin, mi_cap, bp.w1, bp.a_pad, b.cin, bp.b1, m->t1, bp.a_pad, EPI_BIAS_RELU_F16,
                         m->status);
       if (st != ELASTO_OK) return st;
-      st = gemm_plan(&bp.conv2, m->col, mo_cap, bp.w2, bp.b_pad, 9 * bp.a_pad, bp.b2, m->t2, bp.b_pad,
-                        EPI_BIAS_RELU_F16, m->status);
+      st = gemm_plan_conv(&bp.conv2, m->t1, Bm, b.hin, b.win, bp.a_pad, 3, b.stride, 1, bp.w2, bp.b_pad, bp.b2, m->t2,
+                          bp.b_pad, EPI_BIAS_RELU_F16, m->status);
       if (st != ELASTO_OK) return st;
       st = gemm_plan(&bp.conv3, m->t2, mo_cap, bp.w3, 4 * b.w, bp.b_pad, bp.b3, xout, 4 * b.w,
                         EPI_BIAS_RESID_RELU_F16, m->status);
       if (st != ELASTO_OK) return st;
-      bp.conv3.args.resid = b.proj ? m->sc : xin;
-      bp.conv3.args.ldr = 4 * b.w;
+      st = gemm_set_residual_source(&bp.conv3, b.proj ? m->sc : xin, mo_cap);
+      if (st != ELASTO_OK) return st;
       cm.macs += int64_t(b.hin) * b.win * bp.a * b.cin + int64_t(b.ho) * b.wo * bp.b * 9 * bp.a +
                  int64_t(b.ho) * b.wo * 4 * b.w * bp.b + (b.proj ? int64_t(b.ho) * b.wo * 4 * b.w * b.cin : 0);
-      cm.launches += 4 + (b.proj ? (b.stride == 1 ? 1 : 2) : 0);
+      cm.launches += 3 + (b.proj ? 1 : 0);
     }
   }
   ELASTO_CUDA_TRY(cudaDeviceSynchronize());
@@ -723,7 +708,8 @@ elasto_status cnn_forward(CnnModel* m, int mode, cudaStream_t s, const void* ima
   const int ms = B * m->h1 * m->w1;
   CNN_LAUNCH(rec(ELASTO_K_IM2COL, -1, ms, kStemKp, 0, 0,
                  double(B) * d.img_h * d.img_w * 3 * img_elt + double(ms) * kStemKp * 2),
-             im2col_launch(images, d.weight_dtype, B, d.img_h, d.img_w, 3, 7, 2, 3, m->h1, m->w1, kStemKp, reinterpret_cast<__half*>(m->col), s));
+             stem_im2col_launch(images, d.weight_dtype, B, d.img_h, d.img_w, m->h1, m->w1,
+                                reinterpret_cast<__half*>(m->col), s));
   CNN_LAUNCH(gemm_record(-1, ms, kStemC, kStemK, false), gemm_launch(m->stem, ms, s));
   {
     const size_t total = size_t(B) * m->hp * m->wp * (kStemC / 8);
@@ -741,17 +727,11 @@ elasto_status cnn_forward(CnnModel* m, int mode, cudaStream_t s, const void* ima
     const F16Buf* xin = (i % 2 == 0) ? m->xa : m->xb;
     const int mi = B * b.hin * b.win, mo = B * b.ho * b.wo;
     CNN_LAUNCH(gemm_record(i, mi, bp.a, b.cin, false), gemm_launch(bp.conv1, mi, s));
-    CNN_LAUNCH(rec(ELASTO_K_IM2COL, i, mo, 9 * bp.a_pad, 0, 0, double(mi) * bp.a_pad * 2 + double(mo) * 9 * bp.a_pad * 2),
-               im2col_launch(m->t1, kSrcF16, B, b.hin, b.win, bp.a_pad, 3, b.stride, 1, b.ho, b.wo, 9 * bp.a_pad,
-                             reinterpret_cast<__half*>(m->col), s));
-    CNN_LAUNCH(gemm_record(i, mo, bp.b, 9 * bp.a, false), gemm_launch(bp.conv2, mo, s));
-    if (b.proj) {
-      if (b.stride != 1)
-        CNN_LAUNCH(rec(ELASTO_K_IM2COL, i, mo, b.cin, 0, 0, double(mo) * b.cin * 4),
-                   im2col_launch(xin, kSrcF16, B, b.hin, b.win, b.cin, 1, b.stride, 0, b.ho, b.wo, b.cin,
-                                 reinterpret_cast<__half*>(m->col), s));
-      CNN_LAUNCH(gemm_record(i, mo, 4 * b.w, b.cin, false), gemm_launch(m->down[i], mo, s));
-    }
+    // implicit GEMMs: A is read from the input activation (gemm_record's
+    // A-bytes term counts the im2col view; the input itself is mi x channels)
+    CNN_LAUNCH(gemm_record(i, mo, bp.b, 9 * bp.a, false), gemm_launch(bp.conv2, B, s));
+    if (b.proj)
+      CNN_LAUNCH(gemm_record(i, mo, 4 * b.w, b.cin, false), gemm_launch(m->down[i], b.stride == 1 ? mo : B, s));
     CNN_LAUNCH(gemm_record(i, mo, 4 * b.w, bp.b, true), gemm_launch(bp.conv3, mo, s));
   }
   const BlockShape& last = m->shapes.back();
@@ -833,12 +813,12 @@ elasto_status cnn_export_packed(CnnModel* m, int mode, int block, int which, voi
     case 3: ELASTO_CUDA_TRY(cudaMemcpy(host_dst, bp.b2, bytes, cudaMemcpyDeviceToHost)); break;
     case 5: ELASTO_CUDA_TRY(cudaMemcpy(host_dst, bp.b3, bytes, cudaMemcpyDeviceToHost)); break;
     case 2: {
-      std::vector<uint16_t> pad(size_t(bp.b) * 9 * bp.a_pad);
+      std::vector<uint16_t> pad(size_t(bp.b) * 9 * bp.a_cp);
       ELASTO_CUDA_TRY(cudaMemcpy(pad.data(), bp.w2, pad.size() * 2, cudaMemcpyDeviceToHost));
       uint16_t* o = static_cast<uint16_t*>(host_dst);
       for (int r = 0; r < bp.b; ++r)
         for (int t = 0; t < 9; ++t)
-          memcpy(o + (size_t(r) * 9 + t) * bp.a, pad.data() + (size_t(r) * 9 + t) * bp.a_pad, size_t(bp.a) * 2);
+          memcpy(o + (size_t(r) * 9 + t) * bp.a, pad.data() + (size_t(r) * 9 + t) * bp.a_cp, size_t(bp.a) * 2);
       break;
     }
     case 4: {

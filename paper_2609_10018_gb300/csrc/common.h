@@ -34,6 +34,11 @@ int num_sms();  // of the current device
 // box {box_inner, box_outer}, 128-byte swizzle, out-of-bounds reads as zero.
 bool encode_tmap_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_stride_bytes,
                     uint32_t box_inner, uint32_t box_outer, bool fp32 = false);
+// 4-D f16 tensor (NHWC activations: dims {C, W, H, B}), byte strides of
+// dims 1..3, box in traversed elements, traversal strides (the box loads
+// ceil(box[i] / elem_strides[i]) elements along dim i), 128-byte swizzle.
+bool encode_tmap_4d(CUtensorMap* tm, const void* base, const uint64_t dims[4], const uint64_t strides_bytes[3],
+                    const uint32_t box[4], const uint32_t elem_strides[4]);
 // 3-D bf16 tensor [d2][d1][d0] with byte strides s1 (between d1 rows) and s2.
 bool encode_tmap_3d(CUtensorMap* tm, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1,
                     uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2);
@@ -58,8 +63,6 @@ struct GemmArgs {
   const float* bias;      // [N] or null
   void* out;              // [*, ldo]
   int ldo;
-  const bf16* resid;      // [M, ldr] (RESID_RELU)
-  int ldr;
   int patches;            // PATCH: patches per image
   int tokens;             // PATCH: tokens per image (patches + 1)
   const float* pos;       // PATCH: [tokens, N]
@@ -69,6 +72,16 @@ struct GemmArgs {
   int b_planes;           // 2: W held as bf16 hi + lo planes (fp32-stored models), both multiplied
   int pair;               // 1: clusters of two CTAs sharing 256-row tiles (tcgen05 cta_group::2)
   int f16;                // 1: A, W, the residual and 16-bit outputs are f16 (the *_F16 epilogues), else bf16
+  // Implicit-GEMM convolution (conv != 0): A is never materialised. An M
+  // tile is a block of bw x bh output pixels of nb images; k-block kb = (tap,
+  // 64-channel group) is loaded straight from the NHWC input by a 4-D TMA
+  // tile at (cg * 64, ox0 * stride - pad + kx, oy0 * stride - pad + ky, b0),
+  // the padding read as zeros; W's K axis is (ky, kx, channel padded to 64).
+  int conv;
+  int cv_ks, cv_stride, cv_pad, cv_cgroups;  // kernel size, stride, padding, 64-channel groups per tap
+  int cv_ho, cv_wo, cv_bw, cv_bh, cv_nb;     // output size and the pixel block of one M tile
+  int cv_batch;                              // images in this launch (set at launch)
+  int cv_a_bytes;                            // bytes one A tile load delivers
 };
 
 struct GemmPlan {
@@ -88,9 +101,16 @@ int gemm_pick_bn(int M, int N, int step = 32, bool pair = false);
 // mantissa bits (used for models stored in fp32); both products accumulate.
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
                         void* out, int ldo, int epi, int* status, const bf16* W_lo = nullptr);
-// Residual epilogue: read the addend from src [M_cap, ldo] fp32 instead of
-// the output (out = src + acc + bias).
-elasto_status gemm_set_residual_source(GemmPlan* p, const float* src, int M_cap);
+// Residual epilogues: read the addend from src [M_cap, ldo] (fp32 for
+// RESID_F32, 16-bit for the RESID_RELU ones) instead of the output
+// (out = src + acc + bias). The 16-bit residual epilogues need it.
+elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap);
+// Implicit-GEMM k x k convolution (stride, padding `pad`) of the f16 NHWC
+// input x [B_cap, H, W, C] (C % 8 == 0) with W [N, k * k * Cp] f16, Cp = C
+// rounded up to 64 (zero columns), out = epi(conv + bias) f16 [B_cap, Ho, Wo,
+// ldo] (EPI_BIAS_RELU_F16 or EPI_BIAS_F16). gemm_launch's M is the batch.
+elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W, int C, int k, int stride, int pad,
+                             const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status);
 // Launch for the first M (<= M_cap) rows.
 cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s);
 cudaError_t gemm_init_attributes();

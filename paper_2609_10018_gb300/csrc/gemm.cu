@@ -23,9 +23,10 @@
 //      TMA tensor store. For the residual, the old rows of X are brought into
 //      the same staging buffer by TMA loads issued several chunks ahead, so
 //      the read-modify-write of X runs at full memory parallelism.
+//      The 16-bit residual + ReLU of the CNN block outputs works the same way.
 //    * the remaining epilogues (fp32 out, patch rows with position
-//      embedding, bf16 residual + ReLU) transpose through padded shared memory
-//      for row-contiguous stores.
+//      embedding) transpose through padded shared memory for row-contiguous
+//      stores.
 //  Every mbarrier wait is bounded; a timeout records ELASTO_ERR_TIMEOUT.
 #include "common.h"
 #include "ptx.cuh"
@@ -70,18 +71,32 @@ __device__ __forceinline__ float gelu(float x) {
 template <int EPI>
 struct EpiTraits {
   static constexpr bool half = EPI == EPI_BIAS_RELU_F16 || EPI == EPI_BIAS_F16 || EPI == EPI_BIAS_RESID_RELU_F16;
+  // 16-bit residual + ReLU (block outputs of the CNN): the residual chunk is
+  // brought into the staging buffer by TMA like the fp32 residual stream
+  static constexpr bool resid16 = EPI == EPI_BIAS_RESID_RELU_BF16 || EPI == EPI_BIAS_RESID_RELU_F16;
   static constexpr bool tma = EPI == EPI_BIAS_BF16 || EPI == EPI_BIAS_GELU_BF16 || EPI == EPI_BIAS_RELU_BF16 ||
-                              EPI == EPI_BIAS_RESID_F32 || EPI == EPI_BIAS_RELU_F16 || EPI == EPI_BIAS_F16;
+                              EPI == EPI_BIAS_RESID_F32 || EPI == EPI_BIAS_RELU_F16 || EPI == EPI_BIAS_F16 ||
+                              resid16;
   static constexpr bool f32 = EPI == EPI_BIAS_RESID_F32;
-  static constexpr bool resid = EPI == EPI_BIAS_RESID_F32;
+  static constexpr bool resid = EPI == EPI_BIAS_RESID_F32 || resid16;
   static constexpr int cw = f32 ? 32 : 64;  // columns per 128-byte staging chunk
 };
 
 template <int EPI>
 __device__ __forceinline__ float epi_act(float v) {
   if constexpr (EPI == EPI_BIAS_GELU_BF16) return gelu(v);
-  if constexpr (EPI == EPI_BIAS_RELU_BF16 || EPI == EPI_BIAS_RELU_F16) return fmaxf(v, 0.0f);
+  if constexpr (EPI == EPI_BIAS_RELU_BF16 || EPI == EPI_BIAS_RELU_F16 || EpiTraits<EPI>::resid16)
+    return fmaxf(v, 0.0f);
   return v;
+}
+
+// One 32-bit word of the epilogue's 16-bit type -> two fp32 values.
+template <int EPI>
+__device__ __forceinline__ float2 unpack_in(uint32_t w) {
+  if constexpr (EpiTraits<EPI>::half)
+    return __half22float2(*reinterpret_cast<const __half2*>(&w));
+  else
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
 }
 
 // Two fp32 values -> one 32-bit word of the epilogue's 16-bit output type.
@@ -110,6 +125,19 @@ __device__ __forceinline__ void load_bias(const float* bias, int col, int N, flo
 #pragma unroll
     for (int j = 0; j < W; ++j) b[j] = (bias && col + j < N) ? __ldg(bias + col + j) : 0.0f;
   }
+}
+
+// Implicit-GEMM convolution: number of M tiles and the pixel block of one.
+__host__ __device__ __forceinline__ int conv_mtiles(const GemmArgs& a) {
+  return ((a.cv_wo + a.cv_bw - 1) / a.cv_bw) * ((a.cv_ho + a.cv_bh - 1) / a.cv_bh) *
+         ((a.cv_batch + a.cv_nb - 1) / a.cv_nb);
+}
+__device__ __forceinline__ void conv_tile(const GemmArgs& a, int mtile, int& b0, int& oy0, int& ox0) {
+  const int tx = (a.cv_wo + a.cv_bw - 1) / a.cv_bw, ty = (a.cv_ho + a.cv_bh - 1) / a.cv_bh;
+  const int r = mtile / tx;
+  ox0 = (mtile - r * tx) * a.cv_bw;
+  oy0 = (r % ty) * a.cv_bh;
+  b0 = (r / ty) * a.cv_nb;
 }
 
 // Walks this CTA's sequence of (tile, chunk) pairs, skipping chunks past N.
@@ -167,7 +195,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int M = args.M, N = args.N, bn = args.bn;
   const int nk = (args.K + BK - 1) / BK;
   constexpr int TM = PAIR ? 2 * BM : BM;  // rows per tile
-  const int mt = (M + TM - 1) / TM, nt = (N + bn - 1) / bn;
+  const int mt = args.conv ? conv_mtiles(args) : (M + TM - 1) / TM, nt = (N + bn - 1) / bn;
   const int tiles = mt * nt;
   const int rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;  // this CTA's row half of a pair tile
   const int t_start = PAIR ? static_cast<int>(cluster_id_x()) : static_cast<int>(blockIdx.x);
@@ -221,9 +249,12 @@ __global__ void __launch_bounds__(THREADS, 1)
       long issued = 0;
       bool ok = true;
       // pair: the even CTA's full barrier counts both CTAs' bytes
-      const uint32_t bytes = PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2) : A_STAGE + NB * bn * BK * 2;
+      const uint32_t bytes =
+          PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2) : (args.conv ? args.cv_a_bytes : A_STAGE) + NB * bn * BK * 2;
       for (int t = t_start; t < tiles && ok; t += t_stride) {
         const int m0 = (t / nt) * TM + rank * BM, n0 = (t % nt) * bn;
+        int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
+        if (args.conv) conv_tile(args, t / nt, cb0, cy0, cx0);
         for (int kb = 0; kb < nk; ++kb) {
           if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
             ok = false;
@@ -242,7 +273,14 @@ __global__ void __launch_bounds__(THREADS, 1)
             continue;
           }
           mbar_expect_tx(&full[stage], bytes);
-          tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
+          if (args.conv) {
+            const int tap = kb / args.cv_cgroups, cg = kb - tap * args.cv_cgroups;
+            const int ky = tap / args.cv_ks, kx = tap - ky * args.cv_ks;
+            tma_load_4d(sA + stage * A_STAGE, &tmA, &full[stage], cg * BK, cx0 * args.cv_stride - args.cv_pad + kx,
+                        cy0 * args.cv_stride - args.cv_pad + ky, cb0);
+          } else {
+            tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
+          }
           tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * BK, n0);
           if constexpr (NB == 2) tma_load_2d(sB + stage * BSTG + B_STAGE, &tmB2, &full[stage], kb * BK, n0);
           ++issued;
@@ -434,6 +472,23 @@ __global__ void __launch_bounds__(THREADS, 1)
               o.w += __uint_as_float(v[4 * j + 3]) + bb[4 * j + 3];
               *p = o;
             }
+          } else if constexpr (TR::resid16) {
+            // the residual's 8 values arrived by TMA into this 16-byte piece
+#pragma unroll
+            for (int j = 0; j < NC; ++j) {
+              uint4* p = reinterpret_cast<uint4*>(rowp + (((NC * g + j) ^ (r & 7)) << 4));
+              const uint4 rv = *p;
+              const uint32_t rw[4] = {rv.x, rv.y, rv.z, rv.w};
+              uint32_t ow[4];
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                const float2 rf = unpack_in<EPI>(rw[i]);
+                ow[i] = pack_out<EPI>(epi_act<EPI>(__uint_as_float(v[8 * j + 2 * i]) + bb[8 * j + 2 * i] + rf.x),
+                                      epi_act<EPI>(__uint_as_float(v[8 * j + 2 * i + 1]) + bb[8 * j + 2 * i + 1] +
+                                                   rf.y));
+              }
+              *p = make_uint4(ow[0], ow[1], ow[2], ow[3]);
+            }
           } else {
 #pragma unroll
             for (int j = 0; j < NC; ++j) {
@@ -457,7 +512,13 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (elected) bulk_wait_read_all();
         named_bar_sync(1, EPI_THREADS);
         if (elected) {
-          tma_store_2d(&tmC, buf, n0 + c * CW, m0);
+          if (args.conv) {
+            int cb0, cy0, cx0;
+            conv_tile(args, t / nt, cb0, cy0, cx0);
+            tma_store_4d(&tmC, buf, n0 + c * CW, cx0, cy0, cb0);
+          } else {
+            tma_store_2d(&tmC, buf, n0 + c * CW, m0);
+          }
           bulk_commit();  // stays in flight while the next chunk is computed
           if constexpr (TR::resid) {
             if (stored > 0 && pf.valid) {
@@ -494,7 +555,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ transpose epilogue
-    // (warps 2-5 only; warps 6-9 have nothing to do here)
+    // (warps 2-5 only; the other epilogue warps have nothing to do here)
     if (warp < 6) {
     const int q = warp & 3;  // TMEM lane quarter this warp may access
     float* st = reinterpret_cast<float*>(sC) + (warp - 2) * EPI_TILE;
@@ -522,7 +583,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) st[lane * EPI_LD + j] = __uint_as_float(r[j]);
         __syncwarp();
-        if constexpr (EPI == EPI_BIAS_F32 || EPI == EPI_PATCH_POS_F32) {
+        {  // EPI_BIAS_F32 or EPI_PATCH_POS_F32
           const int col = n0 + c + lane;
           const bool cok = col < N;
           const float bv = (cok && args.bias) ? args.bias[col] : 0.0f;
@@ -544,34 +605,6 @@ __global__ void __launch_bounds__(THREADS, 1)
                     (st[i * EPI_LD + lane] + bv) + args.pos[static_cast<size_t>(1 + p) * N + col];
               }
             }
-          }
-        } else {
-          // EPI_BIAS_RESID_RELU_BF16 / _F16
-          const int cp = (lane & 15) * 2;
-          const int col = n0 + c + cp;
-          const bool cok = col < N;
-          const float b0 = (cok && args.bias) ? args.bias[col] : 0.0f;
-          const float b1 = (cok && args.bias) ? args.bias[col + 1] : 0.0f;
-          uint32_t* out = static_cast<uint32_t*>(args.out);
-#pragma unroll 4
-          for (int i = 0; i < 16; ++i) {
-            const int rr = 2 * i + (lane >> 4);
-            const int row = row0 + rr;
-            if (!(cok && row < M)) continue;
-            const uint32_t rw =
-                *reinterpret_cast<const uint32_t*>(args.resid + static_cast<size_t>(row) * args.ldr + col);
-            float r0, r1;
-            if constexpr (TR::half) {
-              const float2 rf = __half22float2(*reinterpret_cast<const __half2*>(&rw));
-              r0 = rf.x;
-              r1 = rf.y;
-            } else {
-              r0 = __uint_as_float(rw << 16);
-              r1 = __uint_as_float(rw & 0xffff0000u);
-            }
-            const float v0 = fmaxf(st[rr * EPI_LD + cp] + b0 + r0, 0.0f);
-            const float v1 = fmaxf(st[rr * EPI_LD + cp + 1] + b1 + r1, 0.0f);
-            out[(static_cast<size_t>(row) * args.ldo + col) >> 1] = pack_out<EPI>(v0, v1);
           }
         }
         __syncwarp();
@@ -598,6 +631,7 @@ template <int EPI, int NB, bool PAIR>
 cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   GemmArgs a = p.args;
   a.M = M;
+  a.cv_batch = M;  // implicit convolutions: M counts images
   const int nt = (a.N + a.bn - 1) / a.bn;
   if constexpr (PAIR) {
     static int max_clusters[64] = {0};
@@ -626,7 +660,7 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
     cfg.gridDim = dim3(2 * clusters);
     return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<EPI, NB, true>, p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
   } else {
-    const int tiles = ((M + BM - 1) / BM) * nt;
+    const int tiles = (a.conv ? conv_mtiles(a) : (M + BM - 1) / BM) * nt;
     const int grid = tiles < num_sms() ? tiles : num_sms();
     gemm_tc_kernel<EPI, NB, false><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
     return cudaGetLastError();
@@ -697,9 +731,11 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     return ELASTO_ERR_UNSUPPORTED;
   }
   *p = GemmPlan{};
+  const bool resid16 = epi == EPI_BIAS_RESID_RELU_BF16 || epi == EPI_BIAS_RESID_RELU_F16;
   const bool tma_out = epi == EPI_BIAS_BF16 || epi == EPI_BIAS_GELU_BF16 || epi == EPI_BIAS_RELU_BF16 ||
-                       epi == EPI_BIAS_RESID_F32 || epi == EPI_BIAS_RELU_F16 || epi == EPI_BIAS_F16;
+                       epi == EPI_BIAS_RESID_F32 || epi == EPI_BIAS_RELU_F16 || epi == EPI_BIAS_F16 || resid16;
   const bool f32_out = epi == EPI_BIAS_RESID_F32;
+  const bool has_resid = f32_out || resid16;
   GemmArgs& a = p->args;
   a.f16 = (epi == EPI_BIAS_RELU_F16 || epi == EPI_BIAS_F16 || epi == EPI_BIAS_RESID_RELU_F16) ? 1 : 0;
   a.M = M_cap;
@@ -723,10 +759,10 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     // residual GEMMs: 3 operand stages and 5 staging chunks fetched ahead;
     // the others: 4 stages and 2 staging chunks.
     if (pair) {
-      a.stages = f32_out ? 5 : 6;
+      a.stages = has_resid ? 5 : 6;
       a.cbufs = (POOL - a.stages * (A_STAGE + B_STAGE_PAIR)) / CBUF;
     } else {
-      a.stages = W_lo ? 2 : (f32_out ? 3 : 4);
+      a.stages = W_lo ? 2 : (has_resid ? 3 : 4);
       a.cbufs = (POOL - a.stages * (A_STAGE + a.b_planes * B_STAGE)) / CBUF;
     }
     if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
@@ -763,13 +799,97 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   return ELASTO_OK;
 }
 
-elasto_status gemm_set_residual_source(GemmPlan* p, const float* src, int M_cap) {
-  if (!p || !p->valid || p->epi != EPI_BIAS_RESID_F32 || !src) {
+elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W, int C, int k, int stride, int pad,
+                             const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status) {
+  if (!p || !x || !Wt || !out || B_cap <= 0 || H <= 0 || W <= 0 || C <= 0 || k <= 0 || stride <= 0 || pad < 0 ||
+      N <= 0 || (epi != EPI_BIAS_RELU_F16 && epi != EPI_BIAS_F16)) {
+    set_error("gemm_plan_conv: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int Ho = (H + 2 * pad - k) / stride + 1, Wo = (W + 2 * pad - k) / stride + 1;
+  if (C % 8 != 0 || ldo % 8 != 0 || N % 2 != 0 || N > ldo || Ho <= 0 || Wo <= 0 || stride > 2) {
+    set_error("gemm_plan_conv: needs C and ldo multiples of 8, N even, stride 1 or 2");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  *p = GemmPlan{};
+  GemmArgs& a = p->args;
+  const int cg = (C + BK - 1) / BK;
+  a.M = B_cap;
+  a.N = N;
+  a.K = k * k * cg * BK;
+  a.conv = 1;
+  a.cv_ks = k;
+  a.cv_stride = stride;
+  a.cv_pad = pad;
+  a.cv_cgroups = cg;
+  a.cv_ho = Ho;
+  a.cv_wo = Wo;
+  // pixel block of an M tile: the fewest tiles of at most 128 pixels; whole
+  // images when several fit (then nb images per tile)
+  long best = -1;
+  if (Ho * Wo <= BM / 2) {
+    a.cv_bw = Wo;
+    a.cv_bh = Ho;
+    a.cv_nb = BM / (Ho * Wo);
+    best = (B_cap + a.cv_nb - 1) / a.cv_nb;
+  }
+  for (int bw = 1; bw <= Wo && bw <= BM; ++bw)
+    for (int bh = 1; bh <= Ho && bw * bh <= BM; ++bh) {
+      const long tiles = long((Wo + bw - 1) / bw) * ((Ho + bh - 1) / bh) * B_cap;
+      if (best < 0 || tiles < best || (tiles == best && a.cv_nb == 1 && bw > a.cv_bw)) {
+        best = tiles;
+        a.cv_bw = bw;
+        a.cv_bh = bh;
+        a.cv_nb = 1;
+      }
+    }
+  const int rows = a.cv_bw * a.cv_bh * a.cv_nb;
+  a.cv_a_bytes = rows * BK * 2;
+  a.cv_batch = B_cap;
+  a.bn = gemm_pick_bn(conv_mtiles(a) * BM, N, 64, false);
+  a.bias = bias;
+  a.out = out;
+  a.ldo = ldo;
+  a.status = status;
+  a.b_planes = 1;
+  a.f16 = 1;
+  a.pair = 0;
+  a.stages = 4;
+  a.cbufs = (POOL - a.stages * (A_STAGE + B_STAGE)) / CBUF;
+  if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
+  if (a.cbufs < 2 || rows > BM) {
+    set_error("gemm_plan_conv: shared-memory layout does not fit");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  const uint64_t xd[4] = {uint64_t(C), uint64_t(W), uint64_t(H), uint64_t(B_cap)};
+  const uint64_t xs[3] = {uint64_t(C) * 2, uint64_t(W) * C * 2, uint64_t(H) * W * C * 2};
+  const uint32_t xb[4] = {uint32_t(BK), uint32_t(a.cv_bw * stride), uint32_t(a.cv_bh * stride), uint32_t(a.cv_nb)};
+  const uint32_t xe[4] = {1u, uint32_t(stride), uint32_t(stride), 1u};
+  const uint64_t od[4] = {uint64_t(N), uint64_t(Wo), uint64_t(Ho), uint64_t(B_cap)};
+  const uint64_t os[3] = {uint64_t(ldo) * 2, uint64_t(Wo) * ldo * 2, uint64_t(Ho) * Wo * ldo * 2};
+  const uint32_t ob[4] = {64u, uint32_t(a.cv_bw), uint32_t(a.cv_bh), uint32_t(a.cv_nb)};
+  const uint32_t oe[4] = {1u, 1u, 1u, 1u};
+  if (xb[1] > 256 || xb[2] > 256 || !encode_tmap_4d(&p->tmA, x, xd, xs, xb, xe) ||
+      !encode_tmap_2d(&p->tmB, Wt, a.K, N, uint64_t(a.K) * 2, BK, a.bn) || !encode_tmap_4d(&p->tmC, out, od, os, ob, oe)) {
+    set_error("gemm_plan_conv: cuTensorMapEncodeTiled failed (alignment or size)");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  p->tmR = p->tmC;
+  p->epi = epi;
+  p->valid = true;
+  return ELASTO_OK;
+}
+
+elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap) {
+  const bool f32 = p && p->epi == EPI_BIAS_RESID_F32;
+  const bool r16 = p && (p->epi == EPI_BIAS_RESID_RELU_BF16 || p->epi == EPI_BIAS_RESID_RELU_F16);
+  if (!p || !p->valid || !(f32 || r16) || !src) {
     set_error("gemm_set_residual_source: needs a residual plan and a source");
     return ELASTO_ERR_INVALID_ARG;
   }
   const int ldo = p->args.ldo;
-  if (!encode_tmap_2d(&p->tmR, src, ldo, M_cap, static_cast<uint64_t>(ldo) * 4, 32, BM, true)) {
+  if (!encode_tmap_2d(&p->tmR, src, ldo, M_cap, static_cast<uint64_t>(ldo) * (f32 ? 4 : 2), f32 ? 32 : 64, BM,
+                      f32)) {
     set_error("gemm_set_residual_source: tensor map (alignment or size)");
     return ELASTO_ERR_UNSUPPORTED;
   }

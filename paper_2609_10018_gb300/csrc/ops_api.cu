@@ -22,9 +22,28 @@ elasto_status elasto_op_gemm(void* stream, const void* A, const void* W, const f
   st = gemm_plan(&p, static_cast<const bf16*>(A), M, static_cast<const bf16*>(W), N, K, bias, out, N, epilogue,
                  status_device);
   if (st != ELASTO_OK) return st;
-  p.args.resid = static_cast<const bf16*>(resid);
-  p.args.ldr = N;
+  if (epilogue == ELASTO_EPI_BIAS_RESID_RELU_BF16 || epilogue == ELASTO_EPI_BIAS_RESID_RELU_F16) {
+    st = gemm_set_residual_source(&p, resid, M);
+    if (st != ELASTO_OK) return st;
+  }
   ELASTO_CUDA_TRY(gemm_launch(p, M, static_cast<cudaStream_t>(stream)));
+  return ELASTO_OK;
+}
+
+elasto_status elasto_op_conv2d(void* stream, const void* x, int B, int H, int W, int C, const void* w, int N, int k,
+                               int stride, int pad, const float* bias, int relu, void* out, int* status_device) {
+  clear_error();
+  if (!x || !w || !out || B <= 0 || H <= 0 || W <= 0 || C <= 0 || N <= 0 || k <= 0 || stride <= 0 || pad < 0) {
+    set_error("elasto_op_conv2d: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  elasto_status st = check_device();
+  if (st != ELASTO_OK) return st;
+  GemmPlan p;
+  st = gemm_plan_conv(&p, x, B, H, W, C, k, stride, pad, w, N, bias, out, N, relu ? EPI_BIAS_RELU_F16 : EPI_BIAS_F16,
+                      status_device);
+  if (st != ELASTO_OK) return st;
+  ELASTO_CUDA_TRY(gemm_launch(p, B, static_cast<cudaStream_t>(stream)));
   return ELASTO_OK;
 }
 

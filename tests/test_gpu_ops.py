@@ -186,3 +186,43 @@ def test_attention_full_size_sampled():
         q = bf16_to_f64(qkv[b])
         ref = np.concatenate([ov.attention(q[:, 0, j], q[:, 1, j], q[:, 2, j], 64) for j in range(h)], axis=-1)
         assert np.max(np.abs(got[b] - ref)) <= 1e-2 * np.max(np.abs(ref))
+
+
+CONV_CASES = [
+    # B, H, W, C, N, k, stride, pad, relu
+    (3, 13, 11, 24, 40, 3, 1, 1, True),      # ragged image, channels below one 64-group
+    (2, 15, 15, 64, 128, 3, 2, 1, True),     # stride 2, odd size
+    (5, 7, 7, 136, 48, 1, 2, 0, False),      # strided 1x1 projection, 3 channel groups (ragged)
+    (1, 56, 56, 64, 64, 3, 1, 1, True),      # ResNet-50 stage 1 conv2 at batch 1
+    (40, 2, 2, 512, 512, 3, 1, 1, True),     # whole images per tile (nb > 1)
+    (4, 9, 9, 16, 24, 3, 2, 1, False),       # N below one 64-column chunk, stride 2
+]
+
+
+@pytest.mark.parametrize("B,H,W,C,N,k,stride,pad,relu", CONV_CASES)
+def test_conv2d_implicit_gemm_matches_fp64(B, H, W, C, N, k, stride, pad, relu):
+    import torch
+    from oracle import resnet as orr
+    rng = np.random.default_rng(B * 1000 + H * 10 + C)
+    x = _f16(rng, (B, H, W, C))
+    wt = (rng.standard_normal((N, C, k, k)) * np.sqrt(2.0 / (C * k * k))).astype(np.float16)
+    bias = rng.standard_normal(N).astype(np.float32) * 0.1
+    cp = (C + 63) // 64 * 64
+    packed = np.zeros((N, k, k, cp), np.float16)
+    packed[..., :C] = wt.transpose(0, 2, 3, 1)
+    ref = orr.conv2d(_f16_to_f64(x), wt.astype(np.float64), stride, pad) + bias
+    if relu:
+        ref = np.maximum(ref, 0)
+    Ho, Wo = ref.shape[1], ref.shape[2]
+    out = empty_dev((B, Ho, Wo, N), torch.uint16)
+    out.fill_(0x7E00)  # f16 NaN: every output must be written
+    st = _status()
+    dx, dw, db = dev(x), dev(packed.view(np.uint16)), dev(bias)
+    binding.elasto_op_conv2d(stream_handle(), dx.data_ptr(), B, H, W, C, dw.data_ptr(), N, k, stride, pad,
+                             db.data_ptr(), relu, out.data_ptr(), st.data_ptr())
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    got = _f16_to_f64(out)
+    assert np.all(np.isfinite(got))
+    scale = float(np.max(np.abs(ref)))
+    assert np.all(np.abs(got - ref) <= 2.0 ** -10 * np.abs(ref) + 1e-4 * scale), float(np.max(np.abs(got - ref)))

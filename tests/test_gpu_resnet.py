@@ -166,3 +166,18 @@ def test_resnet_profile_records_and_queries():
         full = model.query(binding.Q_MODE_MACS, 0)
         assert model.query(binding.Q_MODE_MACS, 3) < model.query(binding.Q_MODE_MACS, 1) < full
         assert model.query(binding.Q_PACKED_BYTES, 3) < model.query(binding.Q_PACKED_BYTES, 0)
+
+
+def test_resnet_fp32_stored_weights_and_images():
+    """weight_dtype ELASTO_F32: fp32 images through the stem gather, fp32
+    weights rounded to f16 after BN folding."""
+    cfg = dataclasses.replace(SMALL, dtype=synth.F32)
+    w, tables = synth.make_resnet_weights(cfg), synth.make_resnet_tables(cfg)
+    img = synth.make_images(cfg, 16, seed=3)
+    assert img.dtype == np.float32
+    with binding.ElasticModel.resnet(cfg, w, tables, max_batch=16) as model:
+        x = dev(img)
+        for m in (0, 3):
+            got = _run(model, x, 16, cfg.classes, m)
+            _report(f"resnet50 32px fp32-stored mode {m}", got, resnet_logits(cfg, tables, m, img))
+            assert rel_err(got, resnet_logits(cfg, tables, m, img)) <= TOL
