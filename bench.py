@@ -229,7 +229,8 @@ def main():
     rank, world, local = dist_env()
     torch.cuda.set_device(local)
     if args.resnet_only:
-        print(json.dumps(resnet50_section(torch, binding, synth, load_peaks()[0])))
+        print(json.dumps(resnet50_section(torch, binding, synth, load_peaks()[0], steps=min(args.steps, 20),
+                                          warmup=max(1, min(args.warmup, 3)))))
         return
     dist = None
     if world > 1:
