@@ -346,8 +346,10 @@ def main():
                                      "tflops": tf, "frac_of_bf16_peak": tf / peaks["bf16_tflops"],
                                      "gflop_per_image": 2 * mm / 1e9,
                                      "packed_weight_mb": model.query(binding.Q_PACKED_BYTES, m) / 1e6})
+        line["batch32"] = batch32_per_mode(model, cfg, tables, torch, binding, peaks)
         line["latency"] = batch1_latency(model, cfg, tables, torch, binding, peaks)
         line["mode_switch_us"] = mode_switch(model, cfg, tables, torch, binding)
+        line["mixed_stream"] = mixed_stream(model, cfg, tables, torch, binding, synth)
         line["e2e"] = e2e(model, cfg, images_np, B, args, torch, binding)
         line["cpu_baseline"] = oracle_cpu_baseline(cfg)
     model.close()
@@ -416,6 +418,89 @@ def resnet50_section(torch, binding, synth, peaks, B=128, steps=20, warmup=3):
     out["mode0_kernels"] = kinds
     model.close()
     return out
+
+
+def batch32_per_mode(model, cfg, tables, torch, binding, peaks, B=32, warmup=10, trials=50):
+    """Per mode at batch 32: 10 warm-up + 50 timed back-to-back forwards
+    (eager launches), per-forward CUDA-event latency p50/p99 and images/s."""
+    from paper_2609_10018_gb300 import synth
+    img = torch.from_numpy(synth.make_images(cfg, B, seed=7)).cuda()
+    lg = torch.empty(B, cfg.classes, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    out = []
+    for m in range(len(tables)):
+        model.set_mode(m)
+        for _ in range(warmup):
+            model.forward(sh, img.data_ptr(), B, lg.data_ptr())
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(trials)]
+        torch.cuda.synchronize()
+        for e0, e1 in ev:
+            e0.record(stream)
+            model.forward(sh, img.data_ptr(), B, lg.data_ptr())
+            e1.record(stream)
+        torch.cuda.synchronize()
+        ts = [e0.elapsed_time(e1) for e0, e1 in ev]
+        macs = model.query(binding.Q_MODE_MACS, m)
+        ips = B * trials / (sum(ts) / 1e3)
+        out.append({"mode": m, "batch": B, "images_per_s": ips, "ms_p50": statistics.median(ts),
+                    "ms_p99": float(np.percentile(ts, 99)),
+                    "frac_of_bf16_peak": 2.0 * macs * ips / 1e12 / peaks["bf16_tflops"]})
+    return out
+
+
+def mixed_stream(model, cfg, tables, torch, binding, synth, n_requests=10_000):
+    """Mixed-mode serving stream on the ViT-B weights: n_requests batches
+    whose mode follows the seeded Markov schedule (stay with p = 0.8, else
+    uniform over the other modes, start in mode 0) and whose size is uniform
+    in {1, 8, 32, 128}; enqueued back to back on one stream, set_mode between
+    batches when the mode changes. Per-batch latency = CUDA events around each
+    forward (device time of the batch); images/s = all images / wall time from
+    the first enqueue to the last completion."""
+    modes, batches = synth.make_stream_schedule(n_requests, len(tables), seed=43)
+    Bmax = int(batches.max())
+    img = torch.from_numpy(synth.make_images(cfg, Bmax, seed=42)).cuda()
+    lg = torch.empty(Bmax, cfg.classes, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    for m in range(len(tables)):  # warm every mode once
+        model.set_mode(m)
+        model.forward(sh, img.data_ptr(), Bmax, lg.data_ptr())
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n_requests)]
+    model.set_mode(int(modes[0]))
+    cur = int(modes[0])
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for i in range(n_requests):
+        m, b = int(modes[i]), int(batches[i])
+        if m != cur:
+            model.set_mode(m)
+            cur = m
+        ev[i][0].record(stream)
+        model.forward(sh, img.data_ptr(), b, lg.data_ptr())
+        ev[i][1].record(stream)
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    lat = np.array([e0.elapsed_time(e1) for e0, e1 in ev])
+    switched = np.zeros(n_requests, bool)
+    switched[1:] = modes[1:] != modes[:-1]
+    # switch overhead: batches right after a switch vs same (mode, batch) without one
+    diffs = []
+    for m in range(len(tables)):
+        for b in np.unique(batches):
+            sel = (modes == m) & (batches == b)
+            a, c = lat[sel & switched], lat[sel & ~switched]
+            if len(a) >= 5 and len(c) >= 5:
+                diffs.append((len(a), float(a.mean() - c.mean())))
+    overhead = sum(n * d for n, d in diffs) / max(1, sum(n for n, _ in diffs))
+    per_b = {int(b): {"requests": int((batches == b).sum()), "ms_p50": float(np.median(lat[batches == b])),
+                      "ms_p99": float(np.percentile(lat[batches == b], 99))} for b in np.unique(batches)}
+    return {"requests": n_requests, "images": int(batches.sum()), "switches": int(switched.sum()),
+            "images_per_s": float(batches.sum() / wall), "wall_s": wall,
+            "batch_ms_p50": float(np.median(lat)), "batch_ms_p99": float(np.percentile(lat, 99)),
+            "per_batch_size": per_b, "switch_overhead_us": 1e3 * overhead,
+            "schedule": "Markov over the 5 modes (stay 0.8, else uniform), start mode 0, seed 43; "
+                        "batch uniform in {1, 8, 32, 128}; images seed 42; eager launches, one stream"}
 
 
 def batch1_latency(model, cfg, tables, torch, binding, peaks):

@@ -79,6 +79,8 @@ __global__ void __launch_bounds__(THREADS, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();  // the set-up above overlapped the previous kernel's tail
+  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -301,8 +303,8 @@ cudaError_t attn_launch(const AttnPlan& p, int batch, cudaStream_t s) {
   if (batch <= 0) return cudaSuccess;
   const int items = batch * p.heads;
   const int grid = items < num_sms() ? items : num_sms();
-  attn_tc_kernel<<<grid, THREADS, SMEM_BYTES, s>>>(p.tmQ, p.tmKV, p.out, p.n, p.n_pad, p.heads, items, p.status);
-  return cudaGetLastError();
+  return launch_pdl(attn_tc_kernel, dim3(grid), dim3(THREADS), SMEM_BYTES, s, p.tmQ, p.tmKV, p.out, p.n, p.n_pad,
+                    p.heads, items, p.status);
 }
 
 }  // namespace elasto

@@ -135,45 +135,6 @@ int n_tensors_expected() {
 
 // ---------------------------------------------------------------- kernels
 
-// The stem's gather (7x7, stride 2, padding 3, 3 channels, 152 columns with
-// 5 zero columns): one warp per output pixel, lane l writing columns l, l+32,
-// ..., so each warp store covers 64 contiguous bytes. A lane's (ky, kx, c)
-// are fixed for the whole kernel and computed once.
-template <typename T>
-__global__ void __launch_bounds__(256) stem_im2col_kernel(const T* __restrict__ src, int H, int W, int Ho, int Wo,
-                                                          size_t rows, __half* __restrict__ dst) {
-  constexpr int NK = (kStemKp + 31) / 32;
-  const int lane = threadIdx.x & 31;
-  int dy[NK], dx[NK], dc[NK];
-#pragma unroll
-  for (int i = 0; i < NK; ++i) {
-    const int k = lane + 32 * i;
-    const int tap = k / 3;
-    dc[i] = k - 3 * tap;
-    dy[i] = k < kStemK ? tap / 7 : -1000;  // padding columns read nothing
-    dx[i] = tap - 7 * (tap / 7);
-  }
-  const size_t warps = static_cast<size_t>(gridDim.x) * (blockDim.x >> 5);
-  for (size_t row = static_cast<size_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); row < rows;
-       row += warps) {
-    const int ox = static_cast<int>(row % Wo);
-    const size_t r2 = row / Wo;
-    const int oy = static_cast<int>(r2 % Ho);
-    const size_t b = r2 / Ho;
-    const T* img = src + b * H * W * 3;
-    __half* out = dst + row * kStemKp;
-#pragma unroll
-    for (int i = 0; i < NK; ++i) {
-      const int k = lane + 32 * i;
-      if (k >= kStemKp) break;
-      const int iy = 2 * oy - 3 + dy[i], ix = 2 * ox - 3 + dx[i];
-      float v = 0.0f;
-      if (iy >= 0 && iy < H && ix >= 0 && ix < W) v = static_cast<float>(img[(static_cast<size_t>(iy) * W + ix) * 3 + dc[i]]);
-      out[k] = __float2half_rn(v);
-    }
-  }
-}
-
 __device__ __forceinline__ void unpack8(const uint4& u, float (&f)[8]) {
   const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
@@ -189,10 +150,49 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
+// The stem's gather (7x7, stride 2, padding 3, 3 channels; 147 columns in
+// (ky, kx, c) order padded with zeros to 152 = 19 groups of 8). Thread t
+// writes group t % 19 of output pixel t / 19 as one 16-byte store, so a warp
+// writes 512 contiguous bytes; the 8 source values of a group are at most
+// two image rows apart and mostly adjacent.
+template <typename T>
+__global__ void __launch_bounds__(256) stem_im2col_kernel(const T* __restrict__ src, int H, int W, int Ho, int Wo,
+                                                          size_t rows, uint4* __restrict__ dst) {
+  pdl_wait();
+  pdl_trigger();
+  constexpr int G = kStemKp / 8;
+  const size_t total = rows * G;
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const size_t row = t / G;
+    const int g = static_cast<int>(t - row * G);
+    const int ox = static_cast<int>(row % Wo);
+    const size_t r2 = row / Wo;
+    const int oy = static_cast<int>(r2 % Ho);
+    const size_t b = r2 / Ho;
+    const T* img = src + b * H * W * 3;
+    float v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int k = g * 8 + i;
+      const int tap = k / 3, c = k - 3 * tap;
+      const int ky = tap / 7, kx = tap - 7 * ky;
+      const int iy = 2 * oy - 3 + ky, ix = 2 * ox - 3 + kx;
+      v[i] = (k < kStemK && iy >= 0 && iy < H && ix >= 0 && ix < W)
+                 ? static_cast<float>(img[(static_cast<size_t>(iy) * W + ix) * 3 + c])
+                 : 0.0f;
+    }
+    dst[t] = make_uint4(pack2(v[0], v[1]), pack2(v[2], v[3]), pack2(v[4], v[5]), pack2(v[6], v[7]));
+  }
+}
+
+
 // 3x3 max pool, stride 2, padding 1 (padding cells are skipped, so they
 // never win), f16 NHWC with C % 8 == 0. Exact: the max of f16 values.
 __global__ void maxpool_kernel(const uint4* __restrict__ src, int H, int W, int C8, int Ho, int Wo, size_t total,
                                uint4* __restrict__ dst) {
+  pdl_wait();
+  pdl_trigger();
   for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
        t += static_cast<size_t>(gridDim.x) * blockDim.x) {
     const int c8 = static_cast<int>(t % C8);
@@ -223,6 +223,8 @@ __global__ void maxpool_kernel(const uint4* __restrict__ src, int H, int W, int 
 // Global average pool: dst[b, c] = mean over the HW pixels of src[b, :, c]
 // (f16 in, fp32 sums and result). Item t = b * C8 + c8.
 __global__ void avgpool_kernel(const uint4* __restrict__ src, int HW, int C8, size_t total, float* __restrict__ dst) {
+  pdl_wait();
+  pdl_trigger();
   for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
        t += static_cast<size_t>(gridDim.x) * blockDim.x) {
     const int c8 = static_cast<int>(t % C8);
@@ -247,13 +249,16 @@ __device__ __forceinline__ float warp_sum32(float v) {
   return v;
 }
 
-constexpr int FC_IMGS = 8, FC_CLASSES = 64;
+constexpr int FC_IMGS = 8, FC_CLASSES = 16;
 
 // logits[b, c] = pooled[b, :] . Wf[c, :] + bf[c] in fp32. grid (ceil(B / 8),
-// ceil(C / 64)), 256 threads: each warp takes classes, 8 images at a time.
+// ceil(C / 16)), 256 threads: each warp takes two classes for 8 images; the
+// classifier row is read 4 float4 at a time so several requests are in flight.
 __global__ void __launch_bounds__(256) fc_kernel(const float* __restrict__ pooled, int B, int d,
                                                  const float* __restrict__ Wf, const float* __restrict__ bf, int C,
                                                  float* __restrict__ logits) {
+  pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b0 = blockIdx.x * FC_IMGS;
   const int nimg = min(FC_IMGS, B - b0);
@@ -265,6 +270,7 @@ __global__ void __launch_bounds__(256) fc_kernel(const float* __restrict__ poole
     float acc[FC_IMGS];
 #pragma unroll
     for (int i = 0; i < FC_IMGS; ++i) acc[i] = 0.0f;
+#pragma unroll 4
     for (int c = lane * 4; c < d; c += 128) {
       const float4 wv = *reinterpret_cast<const float4*>(wr + c);
 #pragma unroll
@@ -292,14 +298,13 @@ cudaError_t stem_im2col_launch(const void* images, int dtype, int B, int H, int 
                                cudaStream_t s) {
   const size_t rows = static_cast<size_t>(B) * Ho * Wo;
   if (rows == 0) return cudaSuccess;
-  const size_t blocks = std::min<size_t>((rows + 7) / 8, 16384);
+  const unsigned blocks = grid_for(rows * (kStemKp / 8));
+  uint4* d = reinterpret_cast<uint4*>(dst);
   if (dtype == ELASTO_BF16)
-    stem_im2col_kernel<bf16><<<unsigned(blocks), 256, 0, s>>>(static_cast<const bf16*>(images), H, W, Ho, Wo, rows,
-                                                              dst);
-  else
-    stem_im2col_kernel<float><<<unsigned(blocks), 256, 0, s>>>(static_cast<const float*>(images), H, W, Ho, Wo,
-                                                               rows, dst);
-  return cudaGetLastError();
+    return launch_pdl(stem_im2col_kernel<bf16>, dim3(blocks), dim3(256), 0, s, static_cast<const bf16*>(images), H, W,
+                      Ho, Wo, rows, d);
+  return launch_pdl(stem_im2col_kernel<float>, dim3(blocks), dim3(256), 0, s, static_cast<const float*>(images), H,
+                    W, Ho, Wo, rows, d);
 }
 
 // ---------------------------------------------------------------- host packing
@@ -715,10 +720,9 @@ elasto_status cnn_forward(CnnModel* m, int mode, cudaStream_t s, const void* ima
     const size_t total = size_t(B) * m->hp * m->wp * (kStemC / 8);
     CNN_LAUNCH(rec(ELASTO_K_POOL, -1, B * m->hp * m->wp, kStemC, 0, 0,
                    double(ms) * kStemC * 2 + double(B) * m->hp * m->wp * kStemC * 2),
-               (maxpool_kernel<<<grid_for(total), 256, 0, s>>>(reinterpret_cast<const uint4*>(m->xb), m->h1, m->w1,
-                                                               kStemC / 8, m->hp, m->wp, total,
-                                                               reinterpret_cast<uint4*>(m->xa)),
-                cudaGetLastError()));
+               launch_pdl(maxpool_kernel, dim3(grid_for(total)), dim3(256), 0, s,
+                          reinterpret_cast<const uint4*>(m->xb), m->h1, m->w1, kStemC / 8, m->hp, m->wp, total,
+                          reinterpret_cast<uint4*>(m->xa)));
   }
   const int nblk = static_cast<int>(m->shapes.size());
   for (int i = 0; i < nblk; ++i) {
@@ -740,15 +744,15 @@ elasto_status cnn_forward(CnnModel* m, int mode, cudaStream_t s, const void* ima
   {
     const size_t total = size_t(B) * (cfin / 8);
     CNN_LAUNCH(rec(ELASTO_K_POOL, nblk, B, cfin, 0, 0, double(B) * hw * cfin * 2 + double(B) * cfin * 4),
-               (avgpool_kernel<<<grid_for(total), 256, 0, s>>>(reinterpret_cast<const uint4*>(xfin), hw, cfin / 8,
-                                                               total, m->pooled),
-                cudaGetLastError()));
+               launch_pdl(avgpool_kernel, dim3(grid_for(total)), dim3(256), 0, s, reinterpret_cast<const uint4*>(xfin),
+                          hw, cfin / 8, total, m->pooled));
   }
   {
     dim3 grid((B + FC_IMGS - 1) / FC_IMGS, (C + FC_CLASSES - 1) / FC_CLASSES);
     CNN_LAUNCH(rec(ELASTO_K_HEAD, -1, B, C, cfin, double(B) * C * cfin,
                    double(B) * cfin * 4 + double(C) * cfin * 4 + double(B) * C * 4),
-               (fc_kernel<<<grid, 256, 0, s>>>(m->pooled, B, cfin, m->fc_w, m->fc_b, C, logits), cudaGetLastError()));
+               launch_pdl(fc_kernel, grid, dim3(256), 0, s, static_cast<const float*>(m->pooled), B, cfin,
+                          static_cast<const float*>(m->fc_w), static_cast<const float*>(m->fc_b), C, logits));
   }
   return ELASTO_OK;
 }

@@ -29,6 +29,33 @@ elasto_status cuda_fail(cudaError_t e, const char* what);  // records "<what>: <
 // ---------------------------------------------------------------- device facts
 int num_sms();  // of the current device
 
+// ---------------------------------------------------------------- launches
+// Programmatic dependent launch. A kernel launched with launch_pdl may be
+// scheduled while the kernel before it on the stream is still finishing, so
+// its prologue (barrier set-up, TMEM allocation, descriptor prefetch) overlaps
+// that kernel's tail. Such a kernel calls pdl_wait() before its first access
+// to global memory: it returns once the previous kernel has completed and its
+// writes are visible, so stream order holds for all data. pdl_trigger() lets
+// the next kernel be scheduled (it still waits in its own pdl_wait()).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // ---------------------------------------------------------------- TMA maps
 // 2-D bf16 tensor [outer][inner] (inner contiguous, row stride in bytes),
 // box {box_inner, box_outer}, 128-byte swizzle, out-of-bounds reads as zero.

@@ -119,6 +119,8 @@ template <int VEC>
 __global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g,
                                                         const float* __restrict__ b, bf16* __restrict__ y,
                                                         int rows, float inv_d) {
+  pdl_wait();
+  pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= rows) return;
@@ -175,7 +177,7 @@ cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf1
   const float inv_d = 1.0f / static_cast<float>(d);
   switch (d / 64) {
 #define LN_CASE(V) \
-  case V: layernorm_kernel<V><<<grid, 256, 0, s>>>(x, g, b, y, rows, inv_d); break;
+  case V: return launch_pdl(layernorm_kernel<V>, grid, dim3(256), 0, s, x, g, b, y, rows, inv_d);
     LN_CASE(1) LN_CASE(2) LN_CASE(3) LN_CASE(4) LN_CASE(5) LN_CASE(6) LN_CASE(8) LN_CASE(10) LN_CASE(12)
     LN_CASE(16)
 #undef LN_CASE
@@ -199,6 +201,8 @@ template <typename T>
 __global__ void patchify_kernel(const T* __restrict__ img, int B, int H, int W, int C, int P, bf16* __restrict__ A,
                                 float* __restrict__ X, const float* __restrict__ cls, const float* __restrict__ pos,
                                 int d) {
+  pdl_wait();
+  pdl_trigger();
   const int gw = W / P, np = (H / P) * gw, K = P * P * C;
   const size_t total2 = static_cast<size_t>(B) * np * K / 2;
   const size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
@@ -233,11 +237,10 @@ cudaError_t patchify_launch(const void* images, int img_dtype, int B, int H, int
   const size_t threads = total2 > static_cast<size_t>(B) * d ? total2 : static_cast<size_t>(B) * d;
   const unsigned blocks = static_cast<unsigned>((threads + 255) / 256);
   if (img_dtype == ELASTO_BF16)
-    patchify_kernel<bf16><<<blocks, 256, 0, s>>>(static_cast<const bf16*>(images), B, H, W, C, P, A, X, cls, pos, d);
-  else
-    patchify_kernel<float><<<blocks, 256, 0, s>>>(static_cast<const float*>(images), B, H, W, C, P, A, X, cls, pos,
-                                                  d);
-  return cudaGetLastError();
+    return launch_pdl(patchify_kernel<bf16>, dim3(blocks), dim3(256), 0, s, static_cast<const bf16*>(images), B, H, W,
+                      C, P, A, X, cls, pos, d);
+  return launch_pdl(patchify_kernel<float>, dim3(blocks), dim3(256), 0, s, static_cast<const float*>(images), B, H,
+                    W, C, P, A, X, cls, pos, d);
 }
 
 namespace {
@@ -247,6 +250,8 @@ namespace {
 // contiguous in the NHWC image, so a piece is one aligned 16-byte copy.
 __global__ void patch_rows_vec_kernel(const bf16* __restrict__ img, int B, int H, int W, int C, int P,
                                       uint4* __restrict__ A) {
+  pdl_wait();
+  pdl_trigger();
   const int gw = W / P, np = (H / P) * gw, n = np + 1, K = P * P * C;
   const int row_pieces = K / 8, seg = P * C / 8;  // pieces per A row, per patch row
   const size_t total = static_cast<size_t>(B) * n * row_pieces;
@@ -268,6 +273,8 @@ __global__ void patch_rows_vec_kernel(const bf16* __restrict__ img, int B, int H
 // Generic version (fp32 images or P*C not a multiple of 8): one thread per element.
 template <typename T>
 __global__ void patch_rows_kernel(const T* __restrict__ img, int B, int H, int W, int C, int P, bf16* __restrict__ A) {
+  pdl_wait();
+  pdl_trigger();
   const int gw = W / P, np = (H / P) * gw, n = np + 1, K = P * P * C;
   const size_t total = static_cast<size_t>(B) * n * K;
   for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
@@ -310,16 +317,15 @@ cudaError_t patch_rows_launch(const void* images, int img_dtype, int B, int H, i
   const int n = (H / P) * (W / P) + 1, K = P * P * C;
   if (img_dtype == ELASTO_BF16 && (P * C) % 8 == 0) {
     const size_t total = static_cast<size_t>(B) * n * (K / 8);
-    patch_rows_vec_kernel<<<grid_1d(total), 256, 0, s>>>(static_cast<const bf16*>(images), B, H, W, C, P,
-                                                         reinterpret_cast<uint4*>(A));
-  } else if (img_dtype == ELASTO_BF16) {
-    patch_rows_kernel<bf16><<<grid_1d(static_cast<size_t>(B) * n * K), 256, 0, s>>>(
-        static_cast<const bf16*>(images), B, H, W, C, P, A);
-  } else {
-    patch_rows_kernel<float><<<grid_1d(static_cast<size_t>(B) * n * K), 256, 0, s>>>(
-        static_cast<const float*>(images), B, H, W, C, P, A);
+    return launch_pdl(patch_rows_vec_kernel, dim3(grid_1d(total)), dim3(256), 0, s, static_cast<const bf16*>(images),
+                      B, H, W, C, P, reinterpret_cast<uint4*>(A));
   }
-  return cudaGetLastError();
+  const unsigned blocks = grid_1d(static_cast<size_t>(B) * n * K);
+  if (img_dtype == ELASTO_BF16)
+    return launch_pdl(patch_rows_kernel<bf16>, dim3(blocks), dim3(256), 0, s, static_cast<const bf16*>(images), B, H,
+                      W, C, P, A);
+  return launch_pdl(patch_rows_kernel<float>, dim3(blocks), dim3(256), 0, s, static_cast<const float*>(images), B, H,
+                    W, C, P, A);
 }
 
 cudaError_t token_addend_launch(const float* cls, const float* pos, const float* patch_b, int n, int d, int B,
@@ -332,16 +338,19 @@ cudaError_t token_addend_launch(const float* cls, const float* pos, const float*
 // ---------------------------------------------------------------- classifier
 namespace {
 
-constexpr int HEAD_IMGS = 8;     // class-token rows per CTA
-constexpr int HEAD_CLASSES = 64; // classes per CTA
+constexpr int HEAD_IMGS = 8;      // class-token rows per CTA
+constexpr int HEAD_CLASSES = 16;  // classes per CTA (two per warp)
 
-// grid (ceil(B / 8), ceil(C / 64)), 256 threads: LayerNorm of up to 8 class
-// tokens into shared memory (fp32), then each warp computes 8 classes x 8
-// images of dot products with float4 loads of the classifier rows.
+// grid (ceil(B / 8), ceil(C / 16)), 256 threads: LayerNorm of up to 8 class
+// tokens into shared memory (fp32), then each warp computes 2 classes x 8
+// images of dot products. The classifier row's loads are issued 4 float4 at a
+// time, so a warp has several HBM/L2 requests in flight instead of one.
 __global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, int B, int n, int d,
                                                    const float* __restrict__ g, const float* __restrict__ bta,
                                                    const float* __restrict__ Wh, const float* __restrict__ bh, int C,
                                                    float* __restrict__ logits) {
+  pdl_wait();
+  pdl_trigger();
   extern __shared__ float sy[];  // [HEAD_IMGS][d]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b0 = blockIdx.x * HEAD_IMGS;
@@ -368,6 +377,7 @@ __global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, 
     float acc[HEAD_IMGS];
 #pragma unroll
     for (int i = 0; i < HEAD_IMGS; ++i) acc[i] = 0.0f;
+#pragma unroll 4
     for (int c = lane * 4; c < d; c += 128) {
       const float4 wv = *reinterpret_cast<const float4*>(wr + c);
 #pragma unroll
@@ -392,8 +402,8 @@ cudaError_t head_launch(const float* X, int B, int n, int d, const float* g, con
                         const float* bh, int C, float* logits, cudaStream_t s) {
   if (B <= 0) return cudaSuccess;
   dim3 grid((B + HEAD_IMGS - 1) / HEAD_IMGS, (C + HEAD_CLASSES - 1) / HEAD_CLASSES);
-  head_kernel<<<grid, 256, HEAD_IMGS * d * sizeof(float), s>>>(X, B, n, d, g, b, Wh, bh, C, logits);
-  return cudaGetLastError();
+  return launch_pdl(head_kernel, grid, dim3(256), HEAD_IMGS * d * sizeof(float), s, X, B, n, d, g, b, Wh, bh, C,
+                    logits);
 }
 
 // ---------------------------------------------------------------- packing

@@ -240,6 +240,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_wait();  // everything above overlapped the previous kernel's tail
+  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -638,16 +640,18 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
     int dev = 0;
     cudaGetDevice(&dev);
     cudaLaunchConfig_t cfg{};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // see launch_pdl
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.blockDim = dim3(THREADS);
     cfg.dynamicSmemBytes = SMEM_BYTES;
     cfg.stream = s;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 1;  // the occupancy query sees the cluster shape only
     if (dev >= 0 && dev < 64 && max_clusters[dev] == 0) {
       cfg.gridDim = dim3(2 * (num_sms() / 2));
       int n = 0;
@@ -658,12 +662,13 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
     const int tiles = ((M + 2 * BM - 1) / (2 * BM)) * nt;
     const int clusters = tiles < max_clusters[dev] ? tiles : max_clusters[dev];
     cfg.gridDim = dim3(2 * clusters);
+    cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<EPI, NB, true>, p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
   } else {
     const int tiles = (a.conv ? conv_mtiles(a) : (M + BM - 1) / BM) * nt;
     const int grid = tiles < num_sms() ? tiles : num_sms();
-    gemm_tc_kernel<EPI, NB, false><<<grid, THREADS, SMEM_BYTES, s>>>(p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
-    return cudaGetLastError();
+    return launch_pdl(gemm_tc_kernel<EPI, NB, false>, dim3(grid), dim3(THREADS), SMEM_BYTES, s, p.tmA, p.tmB, p.tmB2,
+                      p.tmC, p.tmR, a);
   }
 }
 
