@@ -487,10 +487,26 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   // rows): X = addend + P W_pe^T, addend = cls + pos[0] on class tokens and
   // pos[t] + b_pe on patch tokens (Section 4.1: N = HW/P^2 patches, n = N + 1).
   ELASTO_CUDA_TRY(token_addend_launch(h->cls, h->pos, h->patch_b, n, D, Bm, h->tok_addend, 0));
-  st = gemm_plan(&h->patch, h->P, Mcap, h->patch_w, D, kpe, nullptr, h->X, D, EPI_BIAS_RESID_F32, h->status,
-                 h->patch_w_lo);
-  if (st != ELASTO_OK) return st;
-  st = gemm_set_residual_source(&h->patch, h->tok_addend, Mcap);
+  // plan variants for 1, 8 and 32 images (those below max_batch) and max_batch
+  h->n_plan_rows = 0;
+  for (int b : {1, 8, 32})
+    if (b < Bm) h->plan_rows[h->n_plan_rows++] = b * n;
+  h->plan_rows[h->n_plan_rows++] = Mcap;
+  // One GemmPlanSet filled with a plan per bucket by `make(plan, rows)`.
+  auto plan_set = [&](GemmPlanSet& set, auto&& make) -> elasto_status {
+    set.n = h->n_plan_rows;
+    for (int i = 0; i < set.n; ++i) {
+      set.rows[i] = h->plan_rows[i];
+      const elasto_status r = make(set.plan[i], set.rows[i]);
+      if (r != ELASTO_OK) return r;
+    }
+    return ELASTO_OK;
+  };
+  st = plan_set(h->patch, [&](GemmPlan& gp, int rows) {
+    elasto_status r = gemm_plan(&gp, h->P, Mcap, h->patch_w, D, kpe, nullptr, h->X, D, EPI_BIAS_RESID_F32,
+                                h->status, h->patch_w_lo, rows);
+    return r != ELASTO_OK ? r : gemm_set_residual_source(&gp, h->tok_addend, Mcap);
+  });
   if (st != ELASTO_OK) return st;
   ELASTO_CUDA_TRY(cudaDeviceSynchronize());
   const int64_t lin_patch = int64_t(np) * D * kpe + int64_t(D) * C;
@@ -504,24 +520,32 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
                  2 * int64_t(n) * D * lp.f;
       vm.launches += 2;  // two LayerNorms
       if (lp.w > 0) {
-        st = gemm_plan(&lp.qkv, h->Y, Mcap, lp.qkv_w, 3 * lp.w, D, lp.qkv_b, h->QKV, 3 * lp.w, EPI_BIAS_BF16,
-                       h->status, lp.qkv_w_lo);
+        st = plan_set(lp.qkv, [&](GemmPlan& gp, int rows) {
+          return gemm_plan(&gp, h->Y, Mcap, lp.qkv_w, 3 * lp.w, D, lp.qkv_b, h->QKV, 3 * lp.w, EPI_BIAS_BF16,
+                           h->status, lp.qkv_w_lo, rows);
+        });
         if (st != ELASTO_OK) return st;
         st = attn_plan(&lp.attn, h->QKV, h->O, Bm, n, lp.w / 64, h->status);
         if (st != ELASTO_OK) return st;
         vm.launches += 2;
       }
-      st = gemm_plan(&lp.proj, h->O, Mcap, lp.proj_w, D, lp.w, h->proj_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
-                     lp.proj_w_lo);
+      st = plan_set(lp.proj, [&](GemmPlan& gp, int rows) {
+        return gemm_plan(&gp, h->O, Mcap, lp.proj_w, D, lp.w, h->proj_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
+                         lp.proj_w_lo, rows);
+      });
       if (st != ELASTO_OK) return st;
       if (lp.f > 0) {
-        st = gemm_plan(&lp.fc1, h->Y, Mcap, lp.fc1_w, lp.f_pad, D, lp.fc1_b, h->H, lp.f_pad, EPI_BIAS_GELU_BF16,
-                       h->status, lp.fc1_w_lo);
+        st = plan_set(lp.fc1, [&](GemmPlan& gp, int rows) {
+          return gemm_plan(&gp, h->Y, Mcap, lp.fc1_w, lp.f_pad, D, lp.fc1_b, h->H, lp.f_pad, EPI_BIAS_GELU_BF16,
+                           h->status, lp.fc1_w_lo, rows);
+        });
         if (st != ELASTO_OK) return st;
         vm.launches += 1;
       }
-      st = gemm_plan(&lp.fc2, h->H, Mcap, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
-                     lp.fc2_w_lo);
+      st = plan_set(lp.fc2, [&](GemmPlan& gp, int rows) {
+        return gemm_plan(&gp, h->H, Mcap, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
+                         lp.fc2_w_lo, rows);
+      });
       if (st != ELASTO_OK) return st;
       vm.launches += 2;
     }
@@ -564,23 +588,23 @@ elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int b
   h->prof.begin();
   ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, M, h->kpe, 0, 0, double(Mp) * h->kpe * img_elt + double(M) * h->kpe * 2),
                 patch_rows_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, s));
-  ELASTO_LAUNCH(gemm_rec(-1, M, D, h->kpe, 4, true), gemm_launch(h->patch, M, s));
+  ELASTO_LAUNCH(gemm_rec(-1, M, D, h->kpe, 4, true), gemm_launch(h->patch.pick(M), M, s));
   const double ln_bytes = double(M) * D * (4 + 2);
   for (int l = 0; l < d.layers; ++l) {
     const VitLayerPack& lp = vm.layers[l];
     ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, D, 0, 0, ln_bytes),
                   layernorm_launch(h->X, h->ln1_w[l], h->ln1_b[l], h->Y, M, D, s));
     if (lp.w > 0) {
-      ELASTO_LAUNCH(gemm_rec(l, M, 3 * lp.w, D, 2, false), gemm_launch(lp.qkv, M, s));
+      ELASTO_LAUNCH(gemm_rec(l, M, 3 * lp.w, D, 2, false), gemm_launch(lp.qkv.pick(M), M, s));
       ELASTO_LAUNCH(make_rec(ELASTO_K_ATTENTION, l, M, lp.w, n, 2.0 * batch * n * n * lp.w,
                              double(M) * lp.w * 2 * 4),
                     attn_launch(lp.attn, batch, s));
     }
-    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.w, 4, true), gemm_launch(lp.proj, M, s));
+    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.w, 4, true), gemm_launch(lp.proj.pick(M), M, s));
     ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, D, 0, 0, ln_bytes),
                   layernorm_launch(h->X, h->ln2_w[l], h->ln2_b[l], h->Y, M, D, s));
-    if (lp.f > 0) ELASTO_LAUNCH(gemm_rec(l, M, lp.f_pad, D, 2, false), gemm_launch(lp.fc1, M, s));
-    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.f_pad, 4, true), gemm_launch(lp.fc2, M, s));
+    if (lp.f > 0) ELASTO_LAUNCH(gemm_rec(l, M, lp.f_pad, D, 2, false), gemm_launch(lp.fc1.pick(M), M, s));
+    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.f_pad, 4, true), gemm_launch(lp.fc2.pick(M), M, s));
   }
   ELASTO_LAUNCH(make_rec(ELASTO_K_HEAD, -1, batch, C, D, double(batch) * C * D,
                          double(batch) * D * 4 + double(C) * D * 4 + double(batch) * C * 4),

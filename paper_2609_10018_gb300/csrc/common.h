@@ -94,7 +94,8 @@ struct GemmArgs {
   int tokens;             // PATCH: tokens per image (patches + 1)
   const float* pos;       // PATCH: [tokens, N]
   int* status;
-  int stages;             // operand ring depth (<= 4)
+  int stages;             // operand ring depth (<= 8)
+  int b_stage;            // bytes of one B stage (both planes; half of B for a CTA pair)
   int cbufs;              // output staging buffers (16 KB each) for the TMA-store epilogues
   int b_planes;           // 2: W held as bf16 hi + lo planes (fp32-stored models), both multiplied
   int pair;               // 1: clusters of two CTAs sharing 256-row tiles (tcgen05 cta_group::2)
@@ -126,8 +127,25 @@ int gemm_pick_bn(int M, int N, int step = 32, bool pair = false);
 // allocated for the plan's life.
 // W_lo (optional): second bf16 plane so that W = W + W_lo carries ~16
 // mantissa bits (used for models stored in fp32); both products accumulate.
+// M_hint (optional, <= M_cap): the row count the tiling is chosen for (the
+// plan still covers M_cap rows); small batches get narrower N tiles, more
+// CTAs and deeper operand rings.
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
-                        void* out, int ldo, int epi, int* status, const bf16* W_lo = nullptr);
+                        void* out, int ldo, int epi, int* status, const bf16* W_lo = nullptr, int M_hint = 0);
+
+// Launch plans of one GEMM for a few batch sizes: the forward picks the plan
+// made for the smallest row count that covers its rows.
+struct GemmPlanSet {
+  static constexpr int kMax = 4;
+  GemmPlan plan[kMax];
+  int rows[kMax] = {};
+  int n = 0;
+  const GemmPlan& pick(int M) const {
+    for (int i = 0; i < n; ++i)
+      if (M <= rows[i]) return plan[i];
+    return plan[n - 1];
+  }
+};
 // Residual epilogues: read the addend from src [M_cap, ldo] (fp32 for
 // RESID_F32, 16-bit for the RESID_RELU ones) instead of the output
 // (out = src + acc + bias). The 16-bit residual epilogues need it.

@@ -39,8 +39,6 @@ constexpr int BM = 128, BK = 64, MAX_STAGES = 8, MAX_BN = 256;
 constexpr int EPI_THREADS = 512;                 // 16 epilogue warps, four per TMEM lane quarter
 constexpr int THREADS = 64 + EPI_THREADS;
 constexpr int A_STAGE = BM * BK * 2;        // 16 KB
-constexpr int B_STAGE = MAX_BN * BK * 2;    // 32 KB
-constexpr int B_STAGE_PAIR = B_STAGE / 2;   // a CTA of a pair holds half of B
 constexpr int CBUF = BM * 128;              // 16 KB staging chunk (128 rows x 128 B)
 constexpr int POOL = 224 * 1024;            // operand ring + staging buffers
 constexpr int MAX_CBUFS = 8;
@@ -178,7 +176,7 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int S = args.stages, E = args.cbufs;
   // NB: 1, or 2 when W is held as a bf16 (hi, lo) pair
-  constexpr int BSTG = PAIR ? B_STAGE_PAIR : NB * B_STAGE;
+  const int BSTG = args.b_stage;  // NB planes of bn rows (bn / 2 rows per CTA of a pair)
   uint8_t* sA = smem;
   uint8_t* sB = smem + S * A_STAGE;
   uint8_t* sC = sB + S * BSTG;  // E staging chunks, or the transpose tiles
@@ -284,7 +282,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
           }
           tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * BK, n0);
-          if constexpr (NB == 2) tma_load_2d(sB + stage * BSTG + B_STAGE, &tmB2, &full[stage], kb * BK, n0);
+          if constexpr (NB == 2) tma_load_2d(sB + stage * BSTG + BSTG / 2, &tmB2, &full[stage], kb * BK, n0);
           ++issued;
           if (++stage == S) {
             stage = 0;
@@ -344,7 +342,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
                      (kb | k) != 0);
               if constexpr (NB == 2)  // low half of the weights: acc += A . W_lo^T
-                tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + B_STAGE + k * 32, 16, 1024),
+                tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + BSTG / 2 + k * 32, 16, 1024),
                        idesc, 1u);
             }
           }
@@ -726,7 +724,7 @@ int gemm_pick_bn(int M, int N, int step, bool pair) {
 }
 
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
-                        void* out, int ldo, int epi, int* status, const bf16* W_lo) {
+                        void* out, int ldo, int epi, int* status, const bf16* W_lo, int M_hint) {
   if (!p || M_cap <= 0 || N <= 0 || K < 0 || !out || (K > 0 && (!A || !W))) {
     set_error("gemm_plan: invalid arguments");
     return ELASTO_ERR_INVALID_ARG;
@@ -750,10 +748,14 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   // 256-row tile and single-plane weights
   // (long reductions only: with K = 768 the per-tile epilogue dominates and
   // a single CTA per tile measured faster)
-  const bool pair = tma_out && !W_lo && M_cap >= 2 * BM && K >= 1536;
+  const int Mt = (M_hint > 0 && M_hint < M_cap) ? M_hint : M_cap;  // rows the tiling is chosen for
+  const bool pair = tma_out && !W_lo && Mt >= 2 * BM && K >= 1536;
   a.pair = pair ? 1 : 0;
   // bf16 staging chunks are 64 columns wide: their tiles are multiples of 64
-  a.bn = gemm_pick_bn(M_cap, N, (tma_out && !f32_out) ? 64 : 32, pair);
+  a.bn = gemm_pick_bn(Mt, N, (tma_out && !f32_out) ? 64 : 32, pair);
+  // one B stage holds exactly the tile's rows (both planes); the freed bytes
+  // become a deeper operand ring for narrow tiles
+  a.b_stage = pair ? (a.bn / 2) * BK * 2 : (W_lo ? 2 : 1) * a.bn * BK * 2;
   a.bias = bias;
   a.out = out;
   a.ldo = ldo;
@@ -763,13 +765,14 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   if (tma_out) {
     // residual GEMMs: 3 operand stages and 5 staging chunks fetched ahead;
     // the others: 4 stages and 2 staging chunks.
-    if (pair) {
-      a.stages = has_resid ? 5 : 6;
-      a.cbufs = (POOL - a.stages * (A_STAGE + B_STAGE_PAIR)) / CBUF;
-    } else {
-      a.stages = W_lo ? 2 : (has_resid ? 3 : 4);
-      a.cbufs = (POOL - a.stages * (A_STAGE + a.b_planes * B_STAGE)) / CBUF;
-    }
+    // residual epilogues keep 5 staging chunks (residual rows fetched
+    // ahead), the others 2; the rest of the pool is operand ring
+    const int keep = has_resid ? 5 : 2;
+    a.stages = (POOL - keep * CBUF) / (A_STAGE + a.b_stage);
+    if (a.stages > MAX_STAGES) a.stages = MAX_STAGES;
+    if (a.stages < 2) a.stages = 2;
+    if (pair) a.stages = has_resid ? 5 : 6;  // tuned for the K >= 1536 reductions
+    a.cbufs = (POOL - a.stages * (A_STAGE + a.b_stage)) / CBUF;
     if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
     if (ldo % 8 != 0 ||
         !encode_tmap_2d(&p->tmC, out, ldo, M_cap, static_cast<uint64_t>(ldo) * (f32_out ? 4 : 2),
@@ -779,12 +782,13 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     }
     p->tmR = p->tmC;  // the residual is read from the output unless redirected
   } else {
-    a.stages = W_lo ? 2 : 4;
+    a.stages = (POOL - 4 * EPI_TILE * 4) / (A_STAGE + a.b_stage);
+    if (a.stages > 4) a.stages = 4;
     a.cbufs = 0;
   }
   {
     // the operand ring, staging chunks (or transpose tiles) must fit the pool
-    const int bstg = pair ? B_STAGE_PAIR : a.b_planes * B_STAGE;
+    const int bstg = a.b_stage;
     const int tail = tma_out ? a.cbufs * CBUF : 4 * EPI_TILE * 4;
     if (a.stages < 2 || a.stages > MAX_STAGES || a.cbufs > MAX_CBUFS || (tma_out && a.cbufs < 2) ||
         a.stages * (A_STAGE + bstg) + tail > POOL) {
@@ -859,10 +863,12 @@ elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W
   a.b_planes = 1;
   a.f16 = 1;
   a.pair = 0;
-  a.stages = 4;
-  a.cbufs = (POOL - a.stages * (A_STAGE + B_STAGE)) / CBUF;
+  a.b_stage = a.bn * BK * 2;
+  a.stages = (POOL - 2 * CBUF) / (A_STAGE + a.b_stage);
+  if (a.stages > MAX_STAGES) a.stages = MAX_STAGES;
+  a.cbufs = (POOL - a.stages * (A_STAGE + a.b_stage)) / CBUF;
   if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
-  if (a.cbufs < 2 || rows > BM) {
+  if (a.cbufs < 2 || rows > BM || a.stages < 2) {
     set_error("gemm_plan_conv: shared-memory layout does not fit");
     return ELASTO_ERR_UNSUPPORTED;
   }

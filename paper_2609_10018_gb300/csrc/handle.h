@@ -21,7 +21,7 @@ struct VitLayerPack {
   bf16* fc2_w = nullptr;
   // low bf16 planes (fp32-stored models only; W = hi + lo)
   bf16 *qkv_w_lo = nullptr, *proj_w_lo = nullptr, *fc1_w_lo = nullptr, *fc2_w_lo = nullptr;
-  GemmPlan qkv, proj, fc1, fc2;
+  GemmPlanSet qkv, proj, fc1, fc2;  // one plan per batch bucket
   AttnPlan attn;
 };
 
@@ -53,7 +53,9 @@ struct elasto_s {
   void* img_stage = nullptr;
   float* logit_stage = nullptr;
   int* status = nullptr;
-  elasto::GemmPlan patch;
+  elasto::GemmPlanSet patch;
+  int plan_rows[elasto::GemmPlanSet::kMax] = {};  // the row counts the plan variants are made for
+  int n_plan_rows = 0;
   std::vector<elasto::VitMode> modes;
   std::atomic<int> cur{0};
   // CNN state lives behind this pointer (null for ViT)
