@@ -346,6 +346,11 @@ def main():
                                      "tflops": tf, "frac_of_bf16_peak": tf / peaks["bf16_tflops"],
                                      "gflop_per_image": 2 * mm / 1e9,
                                      "packed_weight_mb": model.query(binding.Q_PACKED_BYTES, m) / 1e6})
+        views = [model.query(binding.Q_PACKED_BYTES, m) for m in range(len(tables))]
+        line["packing"] = {"prefix_shared": bool(model.query(binding.Q_PREFIX_SHARED)),
+                           "packed_total_mb": model.query(binding.Q_PACKED_TOTAL) / 1e6,
+                           "sum_of_mode_views_mb": sum(views) / 1e6,
+                           "note": "nested kept sets (Eq. 8): one prefix-ordered packed copy serves every mode"}
         line["batch32"] = batch32_per_mode(model, cfg, tables, torch, binding, peaks)
         line["latency"] = batch1_latency(model, cfg, tables, torch, binding, peaks)
         line["mode_switch_us"] = mode_switch(model, cfg, tables, torch, binding)

@@ -109,6 +109,14 @@ typedef struct {
  * tables, copies the weights to one library-owned device arena, packs every
  * mode's kept rows/columns (Eq. 4, 6, 7 as deletion; "pruning metadata" of
  * Section 4.1-4.2) and allocates the activation workspace for max_batch.
+ * ViT: when every layer's kept head sets and MLP channel sets are nested
+ * across the modes (Eq. 8) and every MLP count is a multiple of 8, one packed
+ * copy per layer serves all modes: heads and channels are ordered "kept by the
+ * smallest mode first", each mode computes on a prefix of that copy (packed
+ * memory = the largest mode's, not the sum over modes; ELASTO_Q_PREFIX_SHARED
+ * reports it). Results then match the per-mode packing up to the fp32
+ * summation order of the out-projection and FC2 reductions. Otherwise each
+ * mode gets its own packed copy.
  * Synchronous. Mode 0 is current afterwards. The caller may free all inputs
  * when this returns. Errors: INVALID_ARG, BAD_TABLE, OOM, CUDA, UNSUPPORTED. */
 elasto_status elasto_create(const elasto_model_desc* desc, const elasto_weights* weights,
@@ -175,12 +183,14 @@ const char* elasto_last_error(void);
 /* Introspection: ELASTO_Q_* values. `mode` is used where it applies. */
 enum {
   ELASTO_Q_N_MODES = 0,
-  ELASTO_Q_PACKED_BYTES = 1,     /* device bytes of one mode's packed weights */
+  ELASTO_Q_PACKED_BYTES = 1,     /* device bytes of packed weights one mode's forward reads */
   ELASTO_Q_SHARED_BYTES = 2,     /* device bytes of mode-independent weights */
   ELASTO_Q_WORKSPACE_BYTES = 3,  /* activation workspace for max_batch */
   ELASTO_Q_ARENA_BYTES = 4,      /* total device bytes owned by the handle */
   ELASTO_Q_MODE_MACS = 5,        /* multiply-accumulates per image of the mode */
-  ELASTO_Q_LAUNCHES = 6          /* kernels one forward of the mode launches */
+  ELASTO_Q_LAUNCHES = 6,         /* kernels one forward of the mode launches */
+  ELASTO_Q_PACKED_TOTAL = 7,     /* device bytes of all modes' packed weights together */
+  ELASTO_Q_PREFIX_SHARED = 8     /* 1 if the modes share one prefix-ordered packed copy */
 };
 elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value);
 

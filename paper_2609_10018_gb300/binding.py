@@ -23,6 +23,7 @@ F32, BF16 = 0, 1
 OK, ERR_INVALID_ARG, ERR_BAD_TABLE, ERR_BAD_MODE, ERR_OOM, ERR_CUDA, ERR_UNSUPPORTED, ERR_TIMEOUT = (
     0, -1, -2, -3, -4, -5, -6, -7)
 Q_N_MODES, Q_PACKED_BYTES, Q_SHARED_BYTES, Q_WORKSPACE_BYTES, Q_ARENA_BYTES, Q_MODE_MACS, Q_LAUNCHES = range(7)
+Q_PACKED_TOTAL, Q_PREFIX_SHARED = 7, 8
 EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_BIAS_RESID_F32, EPI_BIAS_F32, EPI_BIAS_RELU_BF16, EPI_BIAS_RESID_RELU_BF16 = range(6)
 EPI_BIAS_RELU_F16, EPI_BIAS_F16, EPI_BIAS_RESID_RELU_F16 = range(6, 9)  # A, W, resid, out in IEEE f16
 

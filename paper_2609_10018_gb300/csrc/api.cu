@@ -219,6 +219,27 @@ elasto_status vit_check_inputs(const elasto_model_desc* d, const elasto_weights*
   return vit_validate_tables(d, modes, n_modes);
 }
 
+// Nested kept sets (Eq. 8: DN_L contains DN_{L-1}): per layer, the modes'
+// sets ordered by size form a chain S_1 <= S_2 <= ... Returns the prefix order
+// S_1 (ascending), then S_2 \ S_1 (ascending), ..., so that every mode's set
+// is a prefix of it; false if some pair of sets is not nested.
+bool nested_order(const std::vector<std::vector<int32_t>>& sets, std::vector<int32_t>* order) {
+  std::vector<int> by_size(sets.size());
+  for (size_t i = 0; i < sets.size(); ++i) by_size[i] = static_cast<int>(i);
+  std::stable_sort(by_size.begin(), by_size.end(),
+                   [&](int a, int b) { return sets[a].size() < sets[b].size(); });
+  order->clear();
+  std::vector<int32_t> prev;
+  for (int i : by_size) {
+    const std::vector<int32_t>& cur = sets[i];  // sorted ascending (validated)
+    if (!std::includes(cur.begin(), cur.end(), prev.begin(), prev.end())) return false;
+    for (int32_t v : cur)
+      if (!std::binary_search(prev.begin(), prev.end(), v)) order->push_back(v);
+    prev = cur;
+  }
+  return true;
+}
+
 elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, const elasto_mode_tables* modes,
                          int n_modes, elasto_s* h) {
   elasto_status st = vit_check_inputs(d, wts, modes, n_modes);
@@ -249,16 +270,70 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   };
   std::vector<std::vector<Off>> offs(n_modes, std::vector<Off>(L));
   int wmax = 0, fmax = 0;
+  // Prefix sharing when every layer's head and MLP sets are nested across the
+  // modes and every MLP count is a multiple of 8 (a prefix then needs no
+  // padding channels): one packed copy per layer instead of one per mode.
+  h->perm_h.assign(L, {});
+  h->perm_f.assign(L, {});
+  bool shared = n_modes > 1;
+  {
+    std::vector<std::vector<std::vector<int32_t>>> hs(L), fs(L);
+    for (int m = 0; m < n_modes; ++m) {
+      for (int l = 0; l < L; ++l) {
+        size_t a = 0, b = 0;
+        for (int k = 0; k < l; ++k) {
+          a += modes[m].n_heads_kept[k];
+          b += modes[m].n_mlp_kept[k];
+        }
+        hs[l].emplace_back(modes[m].heads_kept + a, modes[m].heads_kept + a + modes[m].n_heads_kept[l]);
+        fs[l].emplace_back(modes[m].mlp_kept + b, modes[m].mlp_kept + b + modes[m].n_mlp_kept[l]);
+        if (modes[m].n_mlp_kept[l] % 8 != 0) shared = false;
+      }
+    }
+    for (int l = 0; l < L && shared; ++l)
+      shared = nested_order(hs[l], &h->perm_h[l]) && nested_order(fs[l], &h->perm_f[l]);
+  }
+  h->prefix_shared = shared;
+  struct SharedOff {
+    size_t qkv_w, qkv_b, proj_w, fc1_w, fc1_b, fc2_w, qkv_lo = 0, proj_lo = 0, fc1_lo = 0, fc2_lo = 0;
+  };
+  std::vector<SharedOff> soff(L);
+  const size_t packed_start = bump.off;
+  if (shared) {
+    for (int l = 0; l < L; ++l) {
+      const size_t hw = 64 * h->perm_h[l].size(), ff = h->perm_f[l].size();
+      SharedOff& o = soff[l];
+      o.qkv_w = bump.take(3 * hw * D * 2);
+      o.qkv_b = bump.take(3 * hw * 4);
+      o.proj_w = bump.take(size_t(D) * hw * 2);
+      o.fc1_w = bump.take(ff * D * 2);
+      o.fc1_b = bump.take(ff * 4);
+      o.fc2_w = bump.take(size_t(D) * ff * 2);
+      if (split) {
+        o.qkv_lo = bump.take(3 * hw * D * 2);
+        o.proj_lo = bump.take(size_t(D) * hw * 2);
+        o.fc1_lo = bump.take(ff * D * 2);
+        o.fc2_lo = bump.take(size_t(D) * ff * 2);
+      }
+    }
+  }
   for (int m = 0; m < n_modes; ++m) {
     const size_t start = bump.off;
     h->modes[m].layers.resize(L);
+    size_t view = 0;
     for (int l = 0; l < L; ++l) {
       VitLayerPack& lp = h->modes[m].layers[l];
       lp.w = 64 * modes[m].n_heads_kept[l];
       lp.f = modes[m].n_mlp_kept[l];
       lp.f_pad = (lp.f + 7) / 8 * 8;
+      lp.ld_proj = shared ? 64 * static_cast<int>(h->perm_h[l].size()) : lp.w;
+      lp.ld_fc2 = shared ? static_cast<int>(h->perm_f[l].size()) : lp.f_pad;
       wmax = std::max(wmax, lp.w);
       fmax = std::max(fmax, lp.f_pad);
+      view += (size_t(3) * lp.w * D * 2 + size_t(3) * lp.w * 4 + size_t(D) * lp.w * 2 + size_t(lp.f_pad) * D * 2 +
+               size_t(lp.f_pad) * 4 + size_t(D) * lp.f_pad * 2) +
+              (split ? size_t(3) * lp.w * D * 2 + size_t(D) * lp.w * 2 + size_t(lp.f_pad) * D * 4 : 0);
+      if (shared) continue;
       Off& o = offs[m][l];
       o.qkv_w = bump.take(size_t(3) * lp.w * D * 2);
       o.qkv_b = bump.take(size_t(3) * lp.w * 4);
@@ -273,8 +348,9 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
         o.fc2_lo = bump.take(size_t(D) * lp.f_pad * 2);
       }
     }
-    h->modes[m].packed_bytes = bump.off - start;
+    h->modes[m].packed_bytes = shared ? view : bump.off - start;
   }
+  h->packed_total = bump.off - packed_start;
   const size_t o_patch_lo = split ? bump.take(size_t(D) * kpe * 2) : 0;
   const size_t ws_start = bump.off;
   const size_t rows = size_t(Bm) * n;
@@ -326,6 +402,22 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   for (int m = 0; m < n_modes; ++m)
     for (int l = 0; l < L; ++l) {
       VitLayerPack& lp = h->modes[m].layers[l];
+      if (shared) {  // every mode points at the one copy of the layer
+        const SharedOff& o = soff[l];
+        lp.qkv_w = reinterpret_cast<bf16*>(A + o.qkv_w);
+        lp.qkv_b = reinterpret_cast<float*>(A + o.qkv_b);
+        lp.proj_w = reinterpret_cast<bf16*>(A + o.proj_w);
+        lp.fc1_w = reinterpret_cast<bf16*>(A + o.fc1_w);
+        lp.fc1_b = reinterpret_cast<float*>(A + o.fc1_b);
+        lp.fc2_w = reinterpret_cast<bf16*>(A + o.fc2_w);
+        if (split) {
+          lp.qkv_w_lo = reinterpret_cast<bf16*>(A + o.qkv_lo);
+          lp.proj_w_lo = reinterpret_cast<bf16*>(A + o.proj_lo);
+          lp.fc1_w_lo = reinterpret_cast<bf16*>(A + o.fc1_lo);
+          lp.fc2_w_lo = reinterpret_cast<bf16*>(A + o.fc2_lo);
+        }
+        continue;
+      }
       const Off& o = offs[m][l];
       lp.qkv_w = reinterpret_cast<bf16*>(A + o.qkv_w);
       lp.qkv_b = reinterpret_cast<float*>(A + o.qkv_b);
@@ -414,7 +506,22 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     UP(up_bf16(W(t0 + 2), size_t(3) * D * D, cw));
     if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(3) * D * D, cwl, s));
     UP(up_f32(W(t0 + 3), size_t(3) * D, cb));
-    for (int m = 0; m < n_modes; ++m) {
+    // shared copy: head-interleaved rows {p * 192 + blk * 64 + r} <- {blk * d + perm[p] * 64 + r}
+    const VitLayerPack& sp = h->modes[0].layers[l];  // its pointers are the shared copy's
+    const std::vector<int32_t>& ph = h->perm_h[l];
+    const std::vector<int32_t>& pf = h->perm_f[l];
+    if (shared && !ph.empty()) {
+      idx.clear();
+      for (int32_t j : ph)
+        for (int blk = 0; blk < 3; ++blk)
+          for (int r = 0; r < 64; ++r) idx.push_back(blk * D + j * 64 + r);
+      ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, int(idx.size()), sp.qkv_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, int(idx.size()), sp.qkv_w_lo, s));
+      ELASTO_CUDA_TRY(gather_f32(cb, di, int(idx.size()), sp.qkv_b, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    for (int m = 0; m < n_modes && !shared; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
       if (lp.w == 0) continue;
       size_t ho = 0;
@@ -433,7 +540,16 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     // proj: columns {j * 64 + r}
     UP(up_bf16(W(t0 + 4), size_t(D) * D, cw));
     if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(D) * D, cwl, s));
-    for (int m = 0; m < n_modes; ++m) {
+    if (shared && !ph.empty()) {  // columns {perm[p] * 64 + r}
+      idx.clear();
+      for (int32_t j : ph)
+        for (int r = 0; r < 64; ++r) idx.push_back(j * 64 + r);
+      ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, D, di, int(idx.size()), sp.proj_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, D, di, int(idx.size()), sp.proj_w_lo, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    for (int m = 0; m < n_modes && !shared; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
       if (lp.w == 0) continue;
       size_t ho = 0;
@@ -451,7 +567,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     UP(up_bf16(W(t0 + 8), size_t(F) * D, cw));
     if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(F) * D, cwl, s));
     UP(up_f32(W(t0 + 9), F, cb));
-    for (int m = 0; m < n_modes; ++m) {
+    if (shared && !pf.empty()) {  // rows perm_f
+      ELASTO_CUDA_TRY(cudaMemcpy(di, pf.data(), pf.size() * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, int(pf.size()), sp.fc1_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, int(pf.size()), sp.fc1_w_lo, s));
+      ELASTO_CUDA_TRY(gather_f32(cb, di, int(pf.size()), sp.fc1_b, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    for (int m = 0; m < n_modes && !shared; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
       if (lp.f == 0) continue;
       size_t fo = 0;
@@ -465,7 +588,13 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     // fc2: columns F into [d, f_pad] (padding columns zero)
     UP(up_bf16(W(t0 + 10), size_t(D) * F, cw));
     if (split) ELASTO_CUDA_TRY(convert_to_bf16_lo(raw.p, dt, size_t(D) * F, cwl, s));
-    for (int m = 0; m < n_modes; ++m) {
+    if (shared && !pf.empty()) {  // columns perm_f
+      ELASTO_CUDA_TRY(cudaMemcpy(di, pf.data(), pf.size() * 4, cudaMemcpyHostToDevice));
+      ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, F, di, int(pf.size()), sp.fc2_w, s));
+      if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, F, di, int(pf.size()), sp.fc2_w_lo, s));
+      ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+    }
+    for (int m = 0; m < n_modes && !shared; ++m) {
       VitLayerPack& lp = h->modes[m].layers[l];
       if (lp.f == 0) continue;
       size_t fo = 0;
@@ -525,13 +654,13 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
                            h->status, lp.qkv_w_lo, rows);
         });
         if (st != ELASTO_OK) return st;
-        st = attn_plan(&lp.attn, h->QKV, h->O, Bm, n, lp.w / 64, h->status);
+        st = attn_plan(&lp.attn, h->QKV, h->O, Bm, n, lp.w / 64, h->status, shared);
         if (st != ELASTO_OK) return st;
         vm.launches += 2;
       }
       st = plan_set(lp.proj, [&](GemmPlan& gp, int rows) {
         return gemm_plan(&gp, h->O, Mcap, lp.proj_w, D, lp.w, h->proj_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
-                         lp.proj_w_lo, rows);
+                         lp.proj_w_lo, rows, lp.ld_proj);
       });
       if (st != ELASTO_OK) return st;
       if (lp.f > 0) {
@@ -544,7 +673,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       }
       st = plan_set(lp.fc2, [&](GemmPlan& gp, int rows) {
         return gemm_plan(&gp, h->H, Mcap, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
-                         lp.fc2_w_lo, rows);
+                         lp.fc2_w_lo, rows, lp.ld_fc2);
       });
       if (st != ELASTO_OK) return st;
       vm.launches += 2;
@@ -771,6 +900,8 @@ elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value) {
     case ELASTO_Q_ARENA_BYTES: *value = int64_t(h->arena_bytes); break;
     case ELASTO_Q_MODE_MACS: *value = h->modes[mode].macs; break;
     case ELASTO_Q_LAUNCHES: *value = h->modes[mode].launches; break;
+    case ELASTO_Q_PACKED_TOTAL: *value = int64_t(h->packed_total); break;
+    case ELASTO_Q_PREFIX_SHARED: *value = h->prefix_shared ? 1 : 0; break;
     default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
   }
   return ELASTO_OK;
@@ -826,6 +957,41 @@ elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int wh
     return ELASTO_ERR_INVALID_ARG;
   }
   if (need == 0) return ELASTO_OK;
+  if (h->prefix_shared) {
+    // The mode's heads / channels are the first k entries of the layer's
+    // prefix order; the export lists them ascending (and q | k | v blocks
+    // apart), so copy the prefix and permute on the host (exact).
+    const bool heads = which <= 2;
+    const std::vector<int32_t>& perm = heads ? h->perm_h[layer] : h->perm_f[layer];
+    const int k = heads ? lp.w / 64 : lp.f;
+    std::vector<int> pos(k);  // pos[q] = prefix position of the q-th smallest kept index
+    for (int i = 0; i < k; ++i) pos[i] = i;
+    std::sort(pos.begin(), pos.end(), [&](int a, int b) { return perm[a] < perm[b]; });
+    const size_t es = (which == 1 || which == 4) ? 4 : 2;
+    std::vector<char> tmp;
+    char* out = static_cast<char*>(host_dst);
+    if (which == 0 || which == 1) {  // rows (or entries) p * 192 + blk * 64 + r -> (blk * k + q) * 64 + r
+      const size_t row = which == 0 ? D * 2 : 4;
+      tmp.resize(size_t(3) * lp.w * row);
+      ELASTO_CUDA_TRY(cudaMemcpy(tmp.data(), src, tmp.size(), cudaMemcpyDeviceToHost));
+      for (int blk = 0; blk < 3; ++blk)
+        for (int q = 0; q < k; ++q)
+          memcpy(out + (size_t(blk) * k + q) * 64 * row, tmp.data() + (size_t(pos[q]) * 3 + blk) * 64 * row, 64 * row);
+    } else if (which == 2 || which == 5) {  // [D, ld] columns of the prefix -> [D, k * width]
+      const int width = which == 2 ? 64 : 1, ld = which == 2 ? lp.ld_proj : lp.ld_fc2;
+      tmp.resize(D * size_t(ld) * es);
+      ELASTO_CUDA_TRY(cudaMemcpy(tmp.data(), src, tmp.size(), cudaMemcpyDeviceToHost));
+      for (size_t r = 0; r < D; ++r)
+        for (int q = 0; q < k; ++q)
+          memcpy(out + (r * k + q) * width * es, tmp.data() + (r * ld + size_t(pos[q]) * width) * es, width * es);
+    } else {  // which 3 / 4: rows (or entries) of FC1 in prefix order
+      const size_t row = which == 3 ? D * 2 : 4;
+      tmp.resize(size_t(k) * row);
+      ELASTO_CUDA_TRY(cudaMemcpy(tmp.data(), src, tmp.size(), cudaMemcpyDeviceToHost));
+      for (int q = 0; q < k; ++q) memcpy(out + size_t(q) * row, tmp.data() + size_t(pos[q]) * row, row);
+    }
+    return ELASTO_OK;
+  }
   if (which == 5) {
     // stored [d, f_pad]; export [d, f]
     ELASTO_CUDA_TRY(cudaMemcpy2D(host_dst, size_t(lp.f) * 2, src, size_t(lp.f_pad) * 2, size_t(lp.f) * 2, D,

@@ -3,8 +3,10 @@
 // pack time, so this kernel never sees them).
 //
 // Input: qkv [B, n, 3, h_m, 64] bf16 exactly as the QKV GEMM writes it (q | k |
-// v blocks, kept heads in ascending order). Output: [B, n, h_m * 64] bf16,
-// the heads concatenated in the same order (the K axis of the sliced W^O).
+// v blocks, kept heads in packing order), or [B, n, h_m, 3, 64] when the modes
+// share one prefix-ordered packed copy (each head's q, k, v adjacent, so a
+// prefix of heads is a prefix of columns). Output: [B, n, h_m * 64] bf16, the
+// heads concatenated in the same order (the K axis of the packed W^O).
 //
 // Persistent kernel; a work item is one (image, kept head) and needs at most
 // two 128-query tiles (n <= 256). Roles:
@@ -42,7 +44,8 @@ constexpr int O_COL = 128;
 
 __global__ void __launch_bounds__(THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmKV,
-                   bf16* __restrict__ out, int n, int n_pad, int heads, int items, int* status) {
+                   bf16* __restrict__ out, int n, int n_pad, int heads, int items, int blk_stride,
+                   int head_stride, int* status) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + 2 * SLOT);
@@ -98,10 +101,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         uint8_t* base = smem + slot * SLOT;
         mbar_expect_tx(&kv_full[slot], bytes);
-        tma_load_3d(base, &tmQ, &kv_full[slot], jj * HD, 0, b);
-        if (tiles == 2) tma_load_3d(base + Q_BYTES, &tmQ, &kv_full[slot], jj * HD, QT, b);
-        tma_load_3d(base + 2 * Q_BYTES, &tmKV, &kv_full[slot], w + jj * HD, 0, b);
-        tma_load_3d(base + 2 * Q_BYTES + KV_BYTES, &tmKV, &kv_full[slot], 2 * w + jj * HD, 0, b);
+        const int qx = jj * head_stride;
+        tma_load_3d(base, &tmQ, &kv_full[slot], qx, 0, b);
+        if (tiles == 2) tma_load_3d(base + Q_BYTES, &tmQ, &kv_full[slot], qx, QT, b);
+        tma_load_3d(base + 2 * Q_BYTES, &tmKV, &kv_full[slot], qx + blk_stride, 0, b);
+        tma_load_3d(base + 2 * Q_BYTES + KV_BYTES, &tmKV, &kv_full[slot], qx + 2 * blk_stride, 0, b);
       }
       if (!ok) record_status(status, ELASTO_ERR_TIMEOUT);
       // the last two items' loads have landed before the CTA exits
@@ -272,7 +276,8 @@ cudaError_t attn_init_attributes() {
                               static_cast<int>(SMEM_BYTES));
 }
 
-elasto_status attn_plan(AttnPlan* p, const bf16* qkv, bf16* out, int batch_cap, int n, int heads, int* status) {
+elasto_status attn_plan(AttnPlan* p, const bf16* qkv, bf16* out, int batch_cap, int n, int heads, int* status,
+                        bool interleaved) {
   if (!p || !qkv || !out || batch_cap <= 0 || n <= 0 || heads <= 0) {
     set_error("attention: invalid arguments");
     return ELASTO_ERR_INVALID_ARG;
@@ -287,6 +292,8 @@ elasto_status attn_plan(AttnPlan* p, const bf16* qkv, bf16* out, int batch_cap, 
   p->n = n;
   p->n_pad = (n + 15) / 16 * 16;
   p->heads = heads;
+  p->blk_stride = interleaved ? HD : heads * HD;
+  p->head_stride = interleaved ? 3 * HD : HD;
   p->batch_cap = batch_cap;
   p->status = status;
   const uint64_t cols = static_cast<uint64_t>(3) * heads * HD;
@@ -304,7 +311,7 @@ cudaError_t attn_launch(const AttnPlan& p, int batch, cudaStream_t s) {
   const int items = batch * p.heads;
   const int grid = items < num_sms() ? items : num_sms();
   return launch_pdl(attn_tc_kernel, dim3(grid), dim3(THREADS), SMEM_BYTES, s, p.tmQ, p.tmKV, p.out, p.n, p.n_pad,
-                    p.heads, items, p.status);
+                    p.heads, items, p.blk_stride, p.head_stride, p.status);
 }
 
 }  // namespace elasto

@@ -788,6 +788,13 @@ elasto_status cnn_query(CnnModel* m, int what, int mode, int64_t* value) {
     case ELASTO_Q_ARENA_BYTES: *value = int64_t(m->arena_bytes); break;
     case ELASTO_Q_MODE_MACS: *value = m->modes[mode].macs; break;
     case ELASTO_Q_LAUNCHES: *value = m->modes[mode].launches; break;
+    case ELASTO_Q_PACKED_TOTAL: {
+      int64_t t = 0;
+      for (const CnnMode& cm : m->modes) t += int64_t(cm.packed_bytes);
+      *value = t;
+      break;
+    }
+    case ELASTO_Q_PREFIX_SHARED: *value = 0; break;
     default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
   }
   return ELASTO_OK;

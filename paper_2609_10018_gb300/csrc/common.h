@@ -130,8 +130,11 @@ int gemm_pick_bn(int M, int N, int step = 32, bool pair = false);
 // M_hint (optional, <= M_cap): the row count the tiling is chosen for (the
 // plan still covers M_cap rows); small batches get narrower N tiles, more
 // CTAs and deeper operand rings.
+// ldw (optional, >= K): row stride of W (and W_lo) in elements, when W is the
+// first K columns of a wider matrix (a mode's prefix of a shared packed copy).
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
-                        void* out, int ldo, int epi, int* status, const bf16* W_lo = nullptr, int M_hint = 0);
+                        void* out, int ldo, int epi, int* status, const bf16* W_lo = nullptr, int M_hint = 0,
+                        int ldw = 0);
 
 // Launch plans of one GEMM for a few batch sizes: the forward picks the plan
 // made for the smallest row count that covers its rows.
@@ -166,10 +169,13 @@ struct AttnPlan {
   const bf16* qkv;
   bf16* out;
   int n, n_pad, heads, batch_cap;
+  int blk_stride, head_stride;  // column of (q|k|v block b, head j) = b * blk_stride + j * head_stride
   int* status;
   bool valid = false;
 };
-elasto_status attn_plan(AttnPlan* p, const bf16* qkv, bf16* out, int batch_cap, int n, int heads, int* status);
+// interleaved: qkv columns are [head][q|k|v][64] instead of [q|k|v][head][64].
+elasto_status attn_plan(AttnPlan* p, const bf16* qkv, bf16* out, int batch_cap, int n, int heads, int* status,
+                        bool interleaved = false);
 cudaError_t attn_launch(const AttnPlan& p, int batch, cudaStream_t s);
 cudaError_t attn_init_attributes();
 

@@ -724,13 +724,14 @@ int gemm_pick_bn(int M, int N, int step, bool pair) {
 }
 
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
-                        void* out, int ldo, int epi, int* status, const bf16* W_lo, int M_hint) {
+                        void* out, int ldo, int epi, int* status, const bf16* W_lo, int M_hint, int ldw) {
   if (!p || M_cap <= 0 || N <= 0 || K < 0 || !out || (K > 0 && (!A || !W))) {
     set_error("gemm_plan: invalid arguments");
     return ELASTO_ERR_INVALID_ARG;
   }
-  if (K % 8 != 0 || N % 2 != 0) {
-    set_error("gemm: K must be a multiple of 8 and N even");
+  if (ldw <= 0) ldw = K;
+  if (K % 8 != 0 || N % 2 != 0 || ldw < K || ldw % 8 != 0) {
+    set_error("gemm: K and ldw must be multiples of 8 (ldw >= K) and N even");
     return ELASTO_ERR_UNSUPPORTED;
   }
   *p = GemmPlan{};
@@ -798,8 +799,8 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   }
   if (K > 0) {
     if (!encode_tmap_2d(&p->tmA, A, K, M_cap, static_cast<uint64_t>(K) * 2, BK, BM) ||
-        !encode_tmap_2d(&p->tmB, W, K, N, static_cast<uint64_t>(K) * 2, BK, pair ? a.bn / 2 : a.bn) ||
-        (W_lo && !encode_tmap_2d(&p->tmB2, W_lo, K, N, static_cast<uint64_t>(K) * 2, BK, a.bn))) {
+        !encode_tmap_2d(&p->tmB, W, K, N, static_cast<uint64_t>(ldw) * 2, BK, pair ? a.bn / 2 : a.bn) ||
+        (W_lo && !encode_tmap_2d(&p->tmB2, W_lo, K, N, static_cast<uint64_t>(ldw) * 2, BK, a.bn))) {
       set_error("gemm_plan: cuTensorMapEncodeTiled failed (alignment or size)");
       return ELASTO_ERR_UNSUPPORTED;
     }

@@ -13,6 +13,8 @@ struct VitLayerPack {
   int w = 0;       // kept heads * 64
   int f = 0;       // kept MLP channels
   int f_pad = 0;   // f rounded up to a multiple of 8 (zero rows/cols; GELU(0) = 0)
+  int ld_proj = 0; // row stride of proj_w (w, or 64 x heads of the shared copy)
+  int ld_fc2 = 0;  // row stride of fc2_w (f_pad, or the shared copy's channels)
   bf16* qkv_w = nullptr;
   float* qkv_b = nullptr;
   bf16* proj_w = nullptr;
@@ -27,7 +29,7 @@ struct VitLayerPack {
 
 struct VitMode {
   std::vector<VitLayerPack> layers;
-  size_t packed_bytes = 0;
+  size_t packed_bytes = 0;  // bytes of packed weights this mode reads
   int64_t macs = 0;
   int launches = 0;
 };
@@ -57,6 +59,12 @@ struct elasto_s {
   int plan_rows[elasto::GemmPlanSet::kMax] = {};  // the row counts the plan variants are made for
   int n_plan_rows = 0;
   std::vector<elasto::VitMode> modes;
+  // Prefix sharing (nested kept sets, Eq. 8): one packed copy per layer with
+  // heads and MLP channels ordered "kept by the smallest mode first"; every
+  // mode uses a prefix of it. perm_h[l] / perm_f[l] give that order.
+  bool prefix_shared = false;
+  std::vector<std::vector<int32_t>> perm_h, perm_f;
+  size_t packed_total = 0;  // device bytes of all modes' packed weights
   std::atomic<int> cur{0};
   // CNN state lives behind this pointer (null for ViT)
   elasto::CnnModel* cnn = nullptr;

@@ -147,13 +147,13 @@ extern "C" elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const 
       if ((st = gemm_plan(&qkv, Y, M, lp.qkv_w, 3 * lp.w, D, lp.qkv_b, QKV, 3 * lp.w, EPI_BIAS_BF16,
                           h->status, lp.qkv_w_lo)) != ELASTO_OK)
         return st;
-      if ((st = attn_plan(&at, QKV, O, batch, n, lp.w / 64, h->status)) != ELASTO_OK) return st;
+      if ((st = attn_plan(&at, QKV, O, batch, n, lp.w / 64, h->status, h->prefix_shared)) != ELASTO_OK) return st;
       ELASTO_CUDA_TRY(gemm_launch(qkv, M, s));
       ELASTO_CUDA_TRY(attn_launch(at, batch, s));
     }
     GemmPlan proj, fc2;
     if ((st = gemm_plan(&proj, O, M, lp.proj_w, D, lp.w, h->proj_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
-                        lp.proj_w_lo)) != ELASTO_OK)
+                        lp.proj_w_lo, 0, lp.ld_proj)) != ELASTO_OK)
       return st;
     ELASTO_CUDA_TRY(gemm_launch(proj, M, s));
     ELASTO_CUDA_TRY(layernorm_launch(X, h->ln2_w[l], h->ln2_b[l], Y, M, D, s));
@@ -165,7 +165,7 @@ extern "C" elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const 
       ELASTO_CUDA_TRY(gemm_launch(fc1, M, s));
     }
     if ((st = gemm_plan(&fc2, H, M, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
-                        lp.fc2_w_lo)) != ELASTO_OK)
+                        lp.fc2_w_lo, 0, lp.ld_fc2)) != ELASTO_OK)
       return st;
     ELASTO_CUDA_TRY(gemm_launch(fc2, M, s));
   }

@@ -150,11 +150,35 @@ def test_degenerate_and_non_nested_tables():
     tables = [t0, odd] + synth.make_vit_tables(cfg, nested=False)[1:]
     img = synth.make_images(cfg, 6)
     with binding.ElasticModel.vit(cfg, w, tables, max_batch=6) as model:
+        assert model.query(binding.Q_PREFIX_SHARED) == 0  # not nested: one packed copy per mode
         x = dev(img)
         for m, t in enumerate(tables):
             got = _run(model, x, 6, cfg.classes, m)
             ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img)
             assert rel_err(got, ref) <= TOL, m
+
+
+@pytest.mark.parametrize("cfg", [synth.TINY, synth.VIT_S, synth.VIT_B], ids=lambda c: c.name)
+def test_nested_modes_share_one_packed_copy(cfg):
+    """Nested kept sets (Eq. 8): one prefix-ordered copy per layer serves every
+    mode, so the packed weights take the largest mode's memory, not the sum
+    over modes; mode 0 and the smallest mode still match the oracle."""
+    w = synth.make_vit_weights(cfg)
+    wide = ov.widen_all(w)
+    tables = synth.make_vit_tables(cfg)
+    img = synth.make_images(cfg, 4)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=4) as model:
+        assert model.query(binding.Q_PREFIX_SHARED) == 1
+        total = model.query(binding.Q_PACKED_TOTAL)
+        views = [model.query(binding.Q_PACKED_BYTES, m) for m in range(len(tables))]
+        assert views[0] == max(views)
+        assert total <= views[0] + 1024 * 6 * cfg.layers  # alignment slack only
+        assert total < sum(views)
+        x = dev(img)
+        for m in (0, len(tables) - 1):
+            t = tables[m]
+            ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img)
+            assert rel_err(_run(model, x, 4, cfg.classes, m), ref) <= TOL, m
 
 
 def test_batch_limits_and_bad_mode(tiny):
