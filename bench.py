@@ -354,6 +354,15 @@ def main():
         line["batch32"] = batch32_per_mode(model, cfg, tables, torch, binding, peaks)
         line["latency"] = batch1_latency(model, cfg, tables, torch, binding, peaks)
         line["mode_switch_us"] = mode_switch(model, cfg, tables, torch, binding)
+        lut = model.profile_dns(torch.cuda.current_stream().cuda_stream, batch=1, trials=50)
+        nan = float("nan")
+        line["dn_selection"] = {
+            "lut_batch1": lut,
+            "eq10_examples": {  # accuracy unknown (synthetic weights): latency / memory budgets only
+                "no_budget": binding.elasto_select_dn(lut, nan, nan, nan),
+                "memory_le_100MB": binding.elasto_select_dn(lut, nan, 100e6, nan),
+                "latency_le_0.5ms": binding.elasto_select_dn(lut, 0.5, nan, nan)},
+            "note": "elasto_profile_dns (median of 50 eager batch-1 forwards per mode) + elasto_select_dn (Eq. 10)"}
         line["mixed_stream"] = mixed_stream(model, cfg, tables, torch, binding, synth)
         line["e2e"] = e2e(model, cfg, images_np, B, args, torch, binding)
         line["cpu_baseline"] = oracle_cpu_baseline(cfg)

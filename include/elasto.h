@@ -215,6 +215,33 @@ typedef struct {
 elasto_status elasto_profile_enable(elasto_t h, int enable);
 elasto_status elasto_profile_read(elasto_t h, elasto_launch_record* out, int capacity, int* count);
 
+/* Runtime DN selection (Section 4.4, Eq. 10). One look-up-table entry per
+ * mode: latency, memory footprint, computational cost, accuracy. */
+typedef struct {
+  float latency_ms;    /* forward latency at the profiled batch */
+  double memory_bytes; /* device bytes of the weights the mode uses (packed view + shared) */
+  double gflops;       /* 2 x multiply-accumulates per forward at the profiled batch, 1e9 */
+  float accuracy;      /* the caller's measured accuracy in %, NaN when unknown */
+} elasto_dn_profile;
+
+/* Profile every mode of h on this GPU: `trials` timed forwards (after 3
+ * warm-up forwards) of `batch` images from the handle's own buffers on
+ * `stream`, latency = median of CUDA-event durations; memory and FLOPs from
+ * the packed layout. accuracy is set to NaN (the paper measures it offline on
+ * a validation set; the caller fills it in). Restores the current mode.
+ * Synchronous. out: n_modes entries. 1 <= batch <= max_batch, trials >= 1.
+ * Errors: INVALID_ARG, CUDA. */
+elasto_status elasto_profile_dns(elasto_t h, void* stream, int batch, int trials, elasto_dn_profile* out);
+
+/* Eq. 10 over a look-up table: among entries with latency_ms <= max_latency_ms,
+ * memory_bytes <= max_memory_bytes and accuracy >= min_accuracy, the one with
+ * the lowest gflops (ties: lower latency, then lower index). A NaN budget
+ * disables that constraint; an entry with NaN accuracy fails any non-NaN
+ * min_accuracy. Host-only, no CUDA. Writes the index to *mode.
+ * Errors: INVALID_ARG (null, n <= 0), BAD_MODE (no entry satisfies them). */
+elasto_status elasto_select_dn(const elasto_dn_profile* lut, int n, float max_latency_ms, double max_memory_bytes,
+                               float min_accuracy, int* mode);
+
 /* Test hook: copy one packed buffer of (mode, layer) to host_dst (bytes must
  * equal its size). ViT `which`: 0 qkv_w bf16 [3w,d], 1 qkv_b fp32 [3w],
  * 2 proj_w bf16 [d,w], 3 fc1_w bf16 [f,d], 4 fc1_b fp32 [f], 5 fc2_w bf16 [d,f]

@@ -51,6 +51,11 @@ KIND_NAMES = {K_PATCHIFY: "patchify", K_GEMM: "gemm", K_LAYERNORM: "layernorm", 
               K_HEAD: "head", K_IM2COL: "im2col", K_POOL: "pool"}
 
 
+class DnProfile(ctypes.Structure):
+    _fields_ = [("latency_ms", ctypes.c_float), ("memory_bytes", ctypes.c_double), ("gflops", ctypes.c_double),
+                ("accuracy", ctypes.c_float)]
+
+
 class LaunchRecord(ctypes.Structure):
     _fields_ = [("kind", c_int), ("layer", c_int), ("m", c_int), ("n", c_int), ("k", c_int),
                 ("ms", ctypes.c_float), ("macs", ctypes.c_double), ("bytes", ctypes.c_double)]
@@ -87,6 +92,9 @@ def lib() -> ctypes.CDLL:
         "elasto_debug_export_packed": [c_void_p, c_int, c_int, c_int, c_void_p, c_size_t],
         "elasto_profile_enable": [c_void_p, c_int],
         "elasto_profile_read": [c_void_p, ctypes.POINTER(LaunchRecord), c_int, ctypes.POINTER(c_int)],
+        "elasto_profile_dns": [c_void_p, c_void_p, c_int, c_int, ctypes.POINTER(DnProfile)],
+        "elasto_select_dn": [ctypes.POINTER(DnProfile), c_int, ctypes.c_float, ctypes.c_double, ctypes.c_float,
+                             ctypes.POINTER(c_int)],
         "elasto_op_gemm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
                            c_void_p],
         "elasto_op_conv2d": [c_void_p, c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int, c_int, c_int,
@@ -251,6 +259,28 @@ def elasto_profile_read(h: int, capacity: int = 1024) -> List[dict]:
              "ms": r.ms, "macs": r.macs, "bytes": r.bytes} for r in buf[:n.value]]
 
 
+def elasto_profile_dns(h: int, stream: int, batch: int, trials: int, n_modes: int) -> List[dict]:
+    """Measured look-up table of the handle's modes (Eq. 10 inputs)."""
+    buf = (DnProfile * n_modes)()
+    _check(lib().elasto_profile_dns(h, stream, batch, trials, buf), "elasto_profile_dns")
+    return [{"latency_ms": e.latency_ms, "memory_bytes": e.memory_bytes, "gflops": e.gflops,
+             "accuracy": e.accuracy} for e in buf]
+
+
+def elasto_select_dn(lut: Sequence[dict], max_latency_ms: float, max_memory_bytes: float,
+                     min_accuracy: float):
+    """Eq. 10 through the C-ABI; None when no DN satisfies the constraints."""
+    buf = (DnProfile * len(lut))()
+    for i, e in enumerate(lut):
+        buf[i] = DnProfile(e["latency_ms"], e["memory_bytes"], e["gflops"], e["accuracy"])
+    mode = c_int(-1)
+    st = lib().elasto_select_dn(buf, len(lut), max_latency_ms, max_memory_bytes, min_accuracy, ctypes.byref(mode))
+    if st == ERR_BAD_MODE:
+        return None
+    _check(st, "elasto_select_dn")
+    return mode.value
+
+
 def elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status=0) -> None:
     _check(lib().elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status), "elasto_op_gemm")
 
@@ -325,6 +355,9 @@ class ElasticModel:
 
     def profile_read(self) -> List[dict]:
         return elasto_profile_read(self.handle)
+
+    def profile_dns(self, stream: int = 0, batch: int = 1, trials: int = 20) -> List[dict]:
+        return elasto_profile_dns(self.handle, stream, batch, trials, self.n_modes)
 
     def export_packed(self, mode: int, layer: int, which: int, out: np.ndarray) -> np.ndarray:
         return elasto_debug_export_packed(self.handle, mode, layer, which, out)

@@ -13,6 +13,8 @@
 
 #include <algorithm>
 #include <atomic>
+#include <cmath>
+#include <limits>
 #include <memory>
 #include <mutex>
 #include <vector>
@@ -924,6 +926,82 @@ elasto_status elasto_profile_read(elasto_t h, elasto_launch_record* out, int cap
   }
   Profiler& p = h->cnn ? *cnn_profiler(h->cnn) : h->prof;
   return p.read(out, capacity, count);
+}
+
+elasto_status elasto_profile_dns(elasto_t h, void* stream, int batch, int trials, elasto_dn_profile* out) {
+  if (!h || !out || trials < 1) {
+    set_error("elasto_profile_dns: null argument or trials < 1");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (batch < 1 || batch > h->d.max_batch) {
+    set_error("elasto_profile_dns: batch outside [1, max_batch]");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int nm = h->cnn ? cnn_n_modes(h->cnn) : static_cast<int>(h->modes.size());
+  const int saved = h->cur.load(std::memory_order_acquire);
+  void* img = h->cnn ? cnn_image_stage(h->cnn) : h->img_stage;
+  float* logits = h->cnn ? cnn_logit_stage(h->cnn) : h->logit_stage;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  ELASTO_CUDA_TRY(cudaEventCreate(&e0));
+  cudaError_t ce = cudaEventCreate(&e1);
+  if (ce != cudaSuccess) {
+    cudaEventDestroy(e0);
+    return cuda_fail(ce, "cudaEventCreate");
+  }
+  elasto_status st = ELASTO_OK;
+  std::vector<float> ts(trials);
+  for (int m = 0; m < nm && st == ELASTO_OK; ++m) {
+    h->cur.store(m, std::memory_order_release);
+    for (int i = 0; i < 3 && st == ELASTO_OK; ++i) st = elasto_forward(h, stream, img, batch, logits);
+    for (int i = 0; i < trials && st == ELASTO_OK; ++i) {
+      if ((ce = cudaEventRecord(e0, s)) != cudaSuccess) break;
+      st = elasto_forward(h, stream, img, batch, logits);
+      if (st != ELASTO_OK || (ce = cudaEventRecord(e1, s)) != cudaSuccess || (ce = cudaEventSynchronize(e1)) != cudaSuccess ||
+          (ce = cudaEventElapsedTime(&ts[i], e0, e1)) != cudaSuccess)
+        break;
+    }
+    if (st == ELASTO_OK && ce != cudaSuccess) st = cuda_fail(ce, "elasto_profile_dns: timing");
+    if (st != ELASTO_OK) break;
+    std::vector<float> sorted = ts;
+    std::sort(sorted.begin(), sorted.end());
+    int64_t packed = 0, shared = 0, macs = 0;
+    elasto_query(h, ELASTO_Q_PACKED_BYTES, m, &packed);
+    elasto_query(h, ELASTO_Q_SHARED_BYTES, m, &shared);
+    elasto_query(h, ELASTO_Q_MODE_MACS, m, &macs);
+    out[m].latency_ms = sorted[trials / 2];
+    out[m].memory_bytes = double(packed + shared);
+    out[m].gflops = 2.0 * double(macs) * batch / 1e9;
+    out[m].accuracy = std::numeric_limits<float>::quiet_NaN();
+  }
+  h->cur.store(saved, std::memory_order_release);
+  cudaEventDestroy(e0);
+  cudaEventDestroy(e1);
+  return st;
+}
+
+elasto_status elasto_select_dn(const elasto_dn_profile* lut, int n, float max_latency_ms, double max_memory_bytes,
+                               float min_accuracy, int* mode) {
+  if (!lut || !mode || n <= 0) {
+    set_error("elasto_select_dn: null argument or empty table");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  int best = -1;
+  for (int i = 0; i < n; ++i) {
+    const elasto_dn_profile& e = lut[i];
+    if (!std::isnan(max_latency_ms) && !(e.latency_ms <= max_latency_ms)) continue;
+    if (!std::isnan(max_memory_bytes) && !(e.memory_bytes <= max_memory_bytes)) continue;
+    if (!std::isnan(min_accuracy) && !(e.accuracy >= min_accuracy)) continue;  // NaN accuracy fails
+    if (best < 0 || e.gflops < lut[best].gflops ||
+        (e.gflops == lut[best].gflops && e.latency_ms < lut[best].latency_ms))
+      best = i;
+  }
+  if (best < 0) {
+    set_error("elasto_select_dn: no descendant network satisfies the constraints");
+    return ELASTO_ERR_BAD_MODE;
+  }
+  *mode = best;
+  return ELASTO_OK;
 }
 
 elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int which, void* host_dst, size_t bytes) {

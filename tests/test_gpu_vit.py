@@ -196,3 +196,22 @@ def test_batch_limits_and_bad_mode(tiny):
         assert model.mode == 0
         assert model.query(binding.Q_N_MODES) == 2
         assert model.query(binding.Q_PACKED_BYTES, 1) < model.query(binding.Q_PACKED_BYTES, 0)
+
+
+def test_profile_dns_and_select(tiny):
+    """elasto_profile_dns measures each mode on this GPU; Eq. 10 over the
+    measured table picks the cheapest mode meeting the budgets."""
+    cfg, w, wide, tables = tiny
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=8) as model:
+        model.set_mode(1)
+        lut = model.profile_dns(stream_handle(), batch=8, trials=10)
+        assert model.mode == 1  # restored
+        assert len(lut) == 2 and all(e["latency_ms"] > 0 for e in lut)
+        assert all(np.isnan(e["accuracy"]) for e in lut)
+        assert lut[1]["gflops"] < lut[0]["gflops"] and lut[1]["memory_bytes"] < lut[0]["memory_bytes"]
+        assert np.isclose(lut[0]["gflops"], 2 * model.query(binding.Q_MODE_MACS, 0) * 8 / 1e9)
+        nan = float("nan")
+        assert binding.elasto_select_dn(lut, nan, nan, nan) == 1
+        lut[0]["accuracy"], lut[1]["accuracy"] = 80.0, 60.0   # the caller's validation accuracies
+        assert binding.elasto_select_dn(lut, nan, nan, 70.0) == 0
+        assert binding.elasto_select_dn(lut, nan, lut[1]["memory_bytes"], 70.0) is None
