@@ -242,6 +242,26 @@ elasto_status elasto_profile_dns(elasto_t h, void* stream, int batch, int trials
 elasto_status elasto_select_dn(const elasto_dn_profile* lut, int n, float max_latency_ms, double max_memory_bytes,
                                float min_accuracy, int* mode);
 
+/* L1-norm saliency of the Compress stage (Section 4.1: a row's saliency is its
+ * average absolute weight; the least salient rows are masked, Eq. 4, 6, 7),
+ * at the granularity of the kept tables. Computed on the current device from
+ * host weights (same descriptor and tensor order as elasto_create; no mode
+ * tables). A unit's score is the mean of the row averages it owns:
+ * ViT:       scores_a [layers * heads]: head j = its 64 output rows of each of
+ *            W^Q, W^K, W^V and its 64 input columns of W^O;
+ *            scores_b [layers * mlp]: channel c = row c of W1, column c of W2.
+ * ResNet-50: scores_a [sum of block widths]: S_a channel = conv1 output row,
+ *            conv2 input slice; scores_b likewise: S_b channel = conv2 output
+ *            row, conv3 input column. Blocks in order.
+ * Synchronous. Errors: INVALID_ARG, CUDA, OOM. */
+elasto_status elasto_saliency(const elasto_model_desc* desc, const elasto_weights* weights, float* scores_a,
+                              float* scores_b);
+
+/* Kept table from saliency scores: the k highest-scoring of n units (ties:
+ * lower index), written ascending to out[k]. Taking every mode's table from
+ * one ranking makes the modes nested (Eq. 8). Host-only. Errors: INVALID_ARG. */
+elasto_status elasto_topk(const float* scores, int n, int k, int32_t* out);
+
 /* Test hook: copy one packed buffer of (mode, layer) to host_dst (bytes must
  * equal its size). ViT `which`: 0 qkv_w bf16 [3w,d], 1 qkv_b fp32 [3w],
  * 2 proj_w bf16 [d,w], 3 fc1_w bf16 [f,d], 4 fc1_b fp32 [f], 5 fc2_w bf16 [d,f]

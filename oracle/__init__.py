@@ -17,11 +17,13 @@ Everything here is a plain, slow, readable definition in float64:
              dense companions, and the BN-folded packed weights.
 - `counts` : multiply-accumulate counting of what the forward passes compute.
 - `select` : runtime DN selection over a profiled look-up table (Eq. 10).
+- `saliency`: the Compress stage's L1-norm saliency (Section 4.1) and the
+             kept tables it induces.
 
 Inputs in bf16 are uint16 bit patterns and are widened exactly to float64;
 the oracle never rounds after that.
 
-Pinning: see the tests under `tests/test_oracle_*.py` and `tests/test_select_dn.py` (paper figures from
+Pinning: see the tests under `tests/test_oracle_*.py` and `tests/test_select_dn.py`, `tests/test_saliency.py` (paper figures from
 Tables 1-3, library special cases via torch float64, closed forms, identities
 of the method). Parity of the DN outputs against trained weights is unpinned:
 no trained weights or datasets exist here.

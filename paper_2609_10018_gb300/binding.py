@@ -95,6 +95,8 @@ def lib() -> ctypes.CDLL:
         "elasto_profile_dns": [c_void_p, c_void_p, c_int, c_int, ctypes.POINTER(DnProfile)],
         "elasto_select_dn": [ctypes.POINTER(DnProfile), c_int, ctypes.c_float, ctypes.c_double, ctypes.c_float,
                              ctypes.POINTER(c_int)],
+        "elasto_saliency": [ctypes.POINTER(ModelDesc), ctypes.POINTER(Weights), c_void_p, c_void_p],
+        "elasto_topk": [c_void_p, c_int, c_int, c_void_p],
         "elasto_op_gemm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
                            c_void_p],
         "elasto_op_conv2d": [c_void_p, c_void_p, c_int, c_int, c_int, c_int, c_void_p, c_int, c_int, c_int, c_int,
@@ -279,6 +281,38 @@ def elasto_select_dn(lut: Sequence[dict], max_latency_ms: float, max_memory_byte
         return None
     _check(st, "elasto_select_dn")
     return mode.value
+
+
+def elasto_saliency(desc: ModelDesc, tensors: Sequence[np.ndarray], n_a: int, n_b: int):
+    """Compress-stage L1 saliency (scores_a, scores_b) computed on the GPU."""
+    keep = _Keep()
+    w = weights_struct(keep, tensors)
+    a = np.zeros(n_a, np.float32)
+    b = np.zeros(n_b, np.float32)
+    _check(lib().elasto_saliency(ctypes.byref(desc), ctypes.byref(w), a.ctypes.data, b.ctypes.data),
+           "elasto_saliency")
+    return a, b
+
+
+def elasto_topk(scores: np.ndarray, k: int) -> np.ndarray:
+    s = np.ascontiguousarray(scores, dtype=np.float32)
+    out = np.zeros(k, np.int32)
+    _check(lib().elasto_topk(s.ctypes.data, len(s), k, out.ctypes.data), "elasto_topk")
+    return out
+
+
+def saliency_tables_vit(cfg, weights, names=None):
+    """Kept tables for cfg's modes from the GPU saliency: per layer the most
+    salient heads / MLP channels (nested across modes, Eq. 8)."""
+    from . import synth
+    names = names or synth.vit_weight_names(cfg)
+    a, b = elasto_saliency(vit_desc(cfg, 1), [weights[k] for k in names], cfg.layers * cfg.heads,
+                           cfg.layers * cfg.mlp)
+    a = a.reshape(cfg.layers, cfg.heads)
+    b = b.reshape(cfg.layers, cfg.mlp)
+    return [{"heads": [elasto_topk(a[l], kh) for l in range(cfg.layers)],
+             "mlp": [elasto_topk(b[l], kf) for l in range(cfg.layers)]}
+            for kh, kf in zip(cfg.mode_heads, cfg.mode_mlp)]
 
 
 def elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status=0) -> None:
