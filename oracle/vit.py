@@ -22,8 +22,13 @@ Readings where the paper is silent:
   - biases of deleted rows (q, k, v, fc1) are deleted with them; b^O and b2
     are kept whole;
   - LayerNorm eps = 1e-6;
-  - the embedding width d is never pruned (the kept-index tables only cover
-    heads and MLP channels).
+  - embedding-width pruning (Section 4.1: the compress stage also shrinks the
+    hidden size of the LayerNorm and patch-embedding layers) keeps a set E of
+    the d channels in every layer alike (the residual stream has one width):
+    the DN is the ViT of width |E| whose weights are the kept sub-blocks, so
+    each LayerNorm normalises over the kept channels only. Heads keep their
+    width d_i = d / h of the base model (and the 1 / sqrt(d_i) scale). With
+    no embedding table every channel is kept.
 """
 from __future__ import annotations
 
@@ -106,8 +111,9 @@ def patchify(images: np.ndarray, P: int) -> np.ndarray:
 
 def embed(w: dict, cfg, images: np.ndarray) -> np.ndarray:
     """Section 4.1: N = HW/P^2 patches linearly projected to d; n = N + 1 with
-    the class token; plus the position embedding. Returns X0 [B, n, d]."""
-    d = cfg.dim
+    the class token; plus the position embedding. Returns X0 [B, n, d] (d =
+    the rows of patch_w: the kept width after embedding pruning)."""
+    d = w["patch_w"].shape[0]
     patches = patchify(widen(images), cfg.patch)
     t = mm(patches, w["patch_w"].reshape(d, -1).T, "patch") + w["patch_b"]
     B = t.shape[0]
@@ -146,14 +152,45 @@ def vit_forward_dense(w: dict, cfg, images: np.ndarray) -> np.ndarray:
     return classify(w, X)
 
 
-def vit_forward_sliced(w: dict, cfg, heads_kept, mlp_kept, images: np.ndarray) -> np.ndarray:
+def slice_embedding(w: dict, cfg, embed_kept) -> dict:
+    """Embedding-width pruning as deletion: every axis of length d that is the
+    residual-stream width keeps the channels E = embed_kept (ascending). The
+    patch embedding, class token, position embedding, LayerNorm parameters,
+    b^O and b2 keep entries E; W^O and W2 keep output rows E; W^Q, W^K, W^V
+    and W1 keep input columns E; the classifier keeps input columns E. The
+    head axes (rows of W_qkv, columns of W^O) are not embedding channels."""
+    E = np.asarray(embed_kept, dtype=np.int64)
+    out = dict(w)
+    out["patch_w"] = w["patch_w"][E]
+    for k in ("patch_b", "cls", "norm_w", "norm_b"):
+        out[k] = w[k][E]
+    out["pos"] = w["pos"][:, E]
+    out["head_w"] = w["head_w"][:, E]
+    for l in range(cfg.layers):
+        p = f"l{l}."
+        for k in ("ln1_w", "ln1_b", "ln2_w", "ln2_b", "proj_b", "fc2_b"):
+            out[p + k] = w[p + k][E]
+        out[p + "qkv_w"] = w[p + "qkv_w"][:, E]
+        out[p + "fc1_w"] = w[p + "fc1_w"][:, E]
+        out[p + "proj_w"] = w[p + "proj_w"][E]
+        out[p + "fc2_w"] = w[p + "fc2_w"][E]
+    # row-major like the inputs (a column gather is column-major in numpy),
+    # so the matrix products see the same layout as without pruning
+    return {k: np.ascontiguousarray(v) for k, v in out.items()}
+
+
+def vit_forward_sliced(w: dict, cfg, heads_kept, mlp_kept, images: np.ndarray,
+                       embed_kept=None) -> np.ndarray:
     """DN forward (Eq. 2-6 with structured masks applied as deletion).
 
     heads_kept[l]: ascending kept head indices of layer l (subset of [0, h)).
     mlp_kept[l]:   ascending kept MLP hidden channels of layer l.
+    embed_kept:    ascending kept embedding channels (None: all d).
     """
     d, h = cfg.dim, cfg.heads
     di = d // h
+    if embed_kept is not None:
+        w = slice_embedding(w, cfg, embed_kept)
     X = embed(w, cfg, images)
     for l in range(cfg.layers):
         p = f"l{l}."
