@@ -91,9 +91,19 @@ typedef struct {
  * ViT: heads_kept is the concatenation over layers of each layer's kept head
  *   indices (n_heads_kept[l] entries for layer l, 0 <= n <= h); mlp_kept
  *   likewise for MLP hidden channels (0 <= n_mlp_kept[l] <= d_ff).
+ * ViT embedding width (Section 4.1: the compress stage also shrinks the
+ *   hidden size of the LayerNorm and patch-embedding layers): embed_kept
+ *   lists the n_embed_kept kept residual-stream channels, 1 <= n <= dim, the
+ *   same set in every layer; the DN is then the ViT of that width (patch
+ *   embedding, class token and position embedding, LayerNorm parameters, b^O
+ *   and b2 keep those entries; W^O and W2 those output rows; W_qkv, W1 and the
+ *   classifier those input columns; each LayerNorm normalises over the kept
+ *   channels). n_embed_kept == 0 (embed_kept may be NULL) keeps all dim
+ *   channels. A model with any embedding-pruned mode packs every mode
+ *   separately (no prefix sharing).
  * ResNet-50: conv_kept_a / conv_kept_b concatenate, per block, the kept
  *   channels after conv1 (S_a) and after conv2 (S_b), 1 <= n <= width.
- * Unused members may be NULL. */
+ * Unused members may be NULL (and counts 0). */
 typedef struct {
   const int32_t* heads_kept;
   const int32_t* n_heads_kept;
@@ -103,6 +113,8 @@ typedef struct {
   const int32_t* n_conv_a;
   const int32_t* conv_kept_b;
   const int32_t* n_conv_b;
+  const int32_t* embed_kept;
+  int32_t n_embed_kept;
 } elasto_mode_tables;
 
 /* Build an elastic model on the current device: validates descriptor and

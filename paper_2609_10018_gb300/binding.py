@@ -43,7 +43,8 @@ class Weights(ctypes.Structure):
 
 class ModeTables(ctypes.Structure):
     _fields_ = [("heads_kept", P_i32), ("n_heads_kept", P_i32), ("mlp_kept", P_i32), ("n_mlp_kept", P_i32),
-                ("conv_kept_a", P_i32), ("n_conv_a", P_i32), ("conv_kept_b", P_i32), ("n_conv_b", P_i32)]
+                ("conv_kept_a", P_i32), ("n_conv_a", P_i32), ("conv_kept_b", P_i32), ("n_conv_b", P_i32),
+                ("embed_kept", P_i32), ("n_embed_kept", ctypes.c_int32)]
 
 
 K_PATCHIFY, K_GEMM, K_LAYERNORM, K_ATTENTION, K_HEAD, K_IM2COL, K_POOL = range(7)
@@ -162,6 +163,9 @@ def vit_mode_tables(keep: _Keep, tables: Sequence[Dict[str, Sequence[np.ndarray]
         arr[m].n_heads_kept = keep.i32([len(h) for h in heads])
         arr[m].mlp_kept = keep.i32(np.concatenate(mlp) if mlp else [])
         arr[m].n_mlp_kept = keep.i32([len(f) for f in mlp])
+        if t.get("embed") is not None:  # kept embedding channels (absent: all)
+            arr[m].embed_kept = keep.i32(t["embed"])
+            arr[m].n_embed_kept = len(t["embed"])
     return arr
 
 

@@ -192,6 +192,15 @@ elasto_status vit_validate_tables(const elasto_model_desc* d, const elasto_mode_
       ho += nh;
       fo += nf;
     }
+    if (t.n_embed_kept < 0 || t.n_embed_kept > d->dim || (t.n_embed_kept > 0 && !t.embed_kept)) {
+      set_error("elasto_create: mode " + std::to_string(m) + ": embedding table count out of range or null");
+      return ELASTO_ERR_BAD_TABLE;
+    }
+    if (t.n_embed_kept > 0 && !tables_ok(t.embed_kept, t.n_embed_kept, d->dim)) {
+      set_error("elasto_create: mode " + std::to_string(m) +
+                ": kept embedding channels must be strictly increasing and in range");
+      return ELASTO_ERR_BAD_TABLE;
+    }
   }
   return ELASTO_OK;
 }
@@ -277,7 +286,17 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   // padding channels): one packed copy per layer instead of one per mode.
   h->perm_h.assign(L, {});
   h->perm_f.assign(L, {});
-  bool shared = n_modes > 1;
+  // Embedding width per mode (Section 4.1): kept channels first, zero padding
+  // up to a multiple of 64 (the GEMM tile and LayerNorm granularity).
+  bool any_emb = false;
+  for (int m = 0; m < n_modes; ++m) {
+    VitEmbed& em = h->modes[m].emb;
+    em.pruned = modes[m].n_embed_kept > 0 && modes[m].n_embed_kept < D;
+    em.d = em.pruned ? modes[m].n_embed_kept : D;
+    em.d_pad = (em.d + 63) / 64 * 64;
+    any_emb = any_emb || em.pruned;
+  }
+  bool shared = n_modes > 1 && !any_emb;
   {
     std::vector<std::vector<std::vector<int32_t>>> hs(L), fs(L);
     for (int m = 0; m < n_modes; ++m) {
@@ -319,9 +338,28 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       }
     }
   }
+  struct EmbOff {
+    size_t patch_w = 0, patch_lo = 0, patch_b = 0, cls = 0, pos = 0, norm_w = 0, norm_b = 0, head_w = 0;
+    std::vector<size_t> lvec;  // per layer: ln1_w, ln1_b, ln2_w, ln2_b, proj_b, fc2_b
+  };
+  std::vector<EmbOff> eoffs(n_modes);
   for (int m = 0; m < n_modes; ++m) {
     const size_t start = bump.off;
     h->modes[m].layers.resize(L);
+    const VitEmbed& em = h->modes[m].emb;
+    const int Dm = em.d_pad;  // the width every d-axis of this mode's packs has
+    if (em.pruned) {
+      EmbOff& eo = eoffs[m];
+      eo.patch_w = bump.take(size_t(Dm) * kpe * 2);
+      if (split) eo.patch_lo = bump.take(size_t(Dm) * kpe * 2);
+      eo.patch_b = bump.take(size_t(Dm) * 4);
+      eo.cls = bump.take(size_t(Dm) * 4);
+      eo.pos = bump.take(size_t(n) * Dm * 4);
+      eo.norm_w = bump.take(size_t(Dm) * 4);
+      eo.norm_b = bump.take(size_t(Dm) * 4);
+      eo.head_w = bump.take(size_t(C) * Dm * 4);
+      for (int k = 0; k < 6 * L; ++k) eo.lvec.push_back(bump.take(size_t(Dm) * 4));
+    }
     size_t view = 0;
     for (int l = 0; l < L; ++l) {
       VitLayerPack& lp = h->modes[m].layers[l];
@@ -332,22 +370,22 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       lp.ld_fc2 = shared ? static_cast<int>(h->perm_f[l].size()) : lp.f_pad;
       wmax = std::max(wmax, lp.w);
       fmax = std::max(fmax, lp.f_pad);
-      view += (size_t(3) * lp.w * D * 2 + size_t(3) * lp.w * 4 + size_t(D) * lp.w * 2 + size_t(lp.f_pad) * D * 2 +
-               size_t(lp.f_pad) * 4 + size_t(D) * lp.f_pad * 2) +
-              (split ? size_t(3) * lp.w * D * 2 + size_t(D) * lp.w * 2 + size_t(lp.f_pad) * D * 4 : 0);
+      view += (size_t(3) * lp.w * Dm * 2 + size_t(3) * lp.w * 4 + size_t(Dm) * lp.w * 2 + size_t(lp.f_pad) * Dm * 2 +
+               size_t(lp.f_pad) * 4 + size_t(Dm) * lp.f_pad * 2) +
+              (split ? size_t(3) * lp.w * Dm * 2 + size_t(Dm) * lp.w * 2 + size_t(lp.f_pad) * Dm * 4 : 0);
       if (shared) continue;
       Off& o = offs[m][l];
-      o.qkv_w = bump.take(size_t(3) * lp.w * D * 2);
+      o.qkv_w = bump.take(size_t(3) * lp.w * Dm * 2);
       o.qkv_b = bump.take(size_t(3) * lp.w * 4);
-      o.proj_w = bump.take(size_t(D) * lp.w * 2);
-      o.fc1_w = bump.take(size_t(lp.f_pad) * D * 2);
+      o.proj_w = bump.take(size_t(Dm) * lp.w * 2);
+      o.fc1_w = bump.take(size_t(lp.f_pad) * Dm * 2);
       o.fc1_b = bump.take(size_t(lp.f_pad) * 4);
-      o.fc2_w = bump.take(size_t(D) * lp.f_pad * 2);
+      o.fc2_w = bump.take(size_t(Dm) * lp.f_pad * 2);
       if (split) {
-        o.qkv_lo = bump.take(size_t(3) * lp.w * D * 2);
-        o.proj_lo = bump.take(size_t(D) * lp.w * 2);
-        o.fc1_lo = bump.take(size_t(lp.f_pad) * D * 2);
-        o.fc2_lo = bump.take(size_t(D) * lp.f_pad * 2);
+        o.qkv_lo = bump.take(size_t(3) * lp.w * Dm * 2);
+        o.proj_lo = bump.take(size_t(Dm) * lp.w * 2);
+        o.fc1_lo = bump.take(size_t(lp.f_pad) * Dm * 2);
+        o.fc2_lo = bump.take(size_t(Dm) * lp.f_pad * 2);
       }
     }
     h->modes[m].packed_bytes = shared ? view : bump.off - start;
@@ -401,6 +439,43 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   h->img_stage = A + o_img;
   h->logit_stage = reinterpret_cast<float*>(A + o_logit);
   h->status = reinterpret_cast<int*>(A + o_status);
+  for (int m = 0; m < n_modes; ++m) {
+    VitEmbed& em = h->modes[m].emb;
+    if (!em.pruned) {  // the handle's full-width parameters
+      em.patch_w = h->patch_w;
+      em.patch_w_lo = h->patch_w_lo;
+      em.patch_b = h->patch_b;
+      em.cls = h->cls;
+      em.pos = h->pos;
+      em.ln1_w = h->ln1_w;
+      em.ln1_b = h->ln1_b;
+      em.ln2_w = h->ln2_w;
+      em.ln2_b = h->ln2_b;
+      em.proj_b = h->proj_b;
+      em.fc2_b = h->fc2_b;
+      em.norm_w = h->norm_w;
+      em.norm_b = h->norm_b;
+      em.head_w = h->head_w;
+      continue;
+    }
+    const EmbOff& eo = eoffs[m];
+    em.patch_w = reinterpret_cast<bf16*>(A + eo.patch_w);
+    em.patch_w_lo = split ? reinterpret_cast<bf16*>(A + eo.patch_lo) : nullptr;
+    em.patch_b = reinterpret_cast<float*>(A + eo.patch_b);
+    em.cls = reinterpret_cast<float*>(A + eo.cls);
+    em.pos = reinterpret_cast<float*>(A + eo.pos);
+    em.norm_w = reinterpret_cast<float*>(A + eo.norm_w);
+    em.norm_b = reinterpret_cast<float*>(A + eo.norm_b);
+    em.head_w = reinterpret_cast<float*>(A + eo.head_w);
+    for (int l = 0; l < L; ++l) {
+      em.ln1_w.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 0]));
+      em.ln1_b.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 1]));
+      em.ln2_w.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 2]));
+      em.ln2_b.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 3]));
+      em.proj_b.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 4]));
+      em.fc2_b.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 5]));
+    }
+  }
   for (int m = 0; m < n_modes; ++m)
     for (int l = 0; l < L; ++l) {
       VitLayerPack& lp = h->modes[m].layers[l];
@@ -448,6 +523,23 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   if (split) ELASTO_CUDA_TRY(cudaMalloc(&canon_lo.p, max_mat * 2));
   ELASTO_CUDA_TRY(cudaMalloc(&canon_b.p, size_t(std::max(3 * D, F)) * 4));
   ELASTO_CUDA_TRY(cudaMalloc(&idxbuf.p, size_t(std::max(3 * D, F) + 64) * 4));
+  // embedding-pruned modes: each mode's kept channels padded with -1 to d_pad
+  // (at m * D), and 0, 1, 2, ... for the axes gathered whole
+  DevTemp eidx, iota;
+  const int n_iota = std::max({kpe, n, C});
+  if (any_emb) {
+    std::vector<int32_t> host(size_t(n_modes) * D, -1), io(n_iota);
+    for (int m = 0; m < n_modes; ++m)
+      if (h->modes[m].emb.pruned)
+        std::copy(modes[m].embed_kept, modes[m].embed_kept + modes[m].n_embed_kept, host.begin() + size_t(m) * D);
+    for (int i = 0; i < n_iota; ++i) io[i] = i;
+    ELASTO_CUDA_TRY(cudaMalloc(&eidx.p, host.size() * 4));
+    ELASTO_CUDA_TRY(cudaMalloc(&iota.p, io.size() * 4));
+    ELASTO_CUDA_TRY(cudaMemcpy(eidx.p, host.data(), host.size() * 4, cudaMemcpyHostToDevice));
+    ELASTO_CUDA_TRY(cudaMemcpy(iota.p, io.data(), io.size() * 4, cudaMemcpyHostToDevice));
+  }
+  auto eix = [&](int m) { return static_cast<const int32_t*>(eidx.p) + size_t(m) * D; };
+  const int32_t* iot = static_cast<const int32_t*>(iota.p);
   cudaStream_t s = 0;
 
   auto up_f32 = [&](const void* src, size_t count, float* dst) -> elasto_status {
@@ -490,6 +582,19 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   UP(up_f32(W(base_final + 1), D, h->norm_b));
   UP(up_f32(W(base_final + 2), size_t(C) * D, h->head_w));
   UP(up_f32(W(base_final + 3), C, h->head_b));
+  for (int m = 0; m < n_modes; ++m) {
+    const VitEmbed& em = h->modes[m].emb;
+    if (!em.pruned) continue;
+    const int Dm = em.d_pad;
+    ELASTO_CUDA_TRY(gather2d_bf16(h->patch_w, kpe, eix(m), Dm, iot, kpe, em.patch_w, s));
+    if (split) ELASTO_CUDA_TRY(gather2d_bf16(h->patch_w_lo, kpe, eix(m), Dm, iot, kpe, em.patch_w_lo, s));
+    ELASTO_CUDA_TRY(gather_f32(h->patch_b, eix(m), Dm, em.patch_b, s));
+    ELASTO_CUDA_TRY(gather_f32(h->cls, eix(m), Dm, em.cls, s));
+    ELASTO_CUDA_TRY(gather2d_f32(h->pos, D, iot, n, eix(m), Dm, em.pos, s));
+    ELASTO_CUDA_TRY(gather_f32(h->norm_w, eix(m), Dm, em.norm_w, s));
+    ELASTO_CUDA_TRY(gather_f32(h->norm_b, eix(m), Dm, em.norm_b, s));
+    ELASTO_CUDA_TRY(gather2d_f32(h->head_w, D, iot, C, eix(m), Dm, em.head_w, s));
+  }
 
   std::vector<int32_t> idx;
   for (int l = 0; l < L; ++l) {
@@ -500,6 +605,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     UP(up_f32(W(t0 + 6), D, h->ln2_w[l]));
     UP(up_f32(W(t0 + 7), D, h->ln2_b[l]));
     UP(up_f32(W(t0 + 11), D, h->fc2_b[l]));
+    for (int m = 0; m < n_modes; ++m) {
+      const VitEmbed& em = h->modes[m].emb;
+      if (!em.pruned) continue;
+      const std::pair<const float*, float*> v[6] = {{h->ln1_w[l], em.ln1_w[l]}, {h->ln1_b[l], em.ln1_b[l]},
+                                                     {h->ln2_w[l], em.ln2_w[l]}, {h->ln2_b[l], em.ln2_b[l]},
+                                                     {h->proj_b[l], em.proj_b[l]}, {h->fc2_b[l], em.fc2_b[l]}};
+      for (const auto& pr : v) ELASTO_CUDA_TRY(gather_f32(pr.first, eix(m), em.d_pad, pr.second, s));
+    }
     bf16* cw = static_cast<bf16*>(canon.p);
     bf16* cwl = static_cast<bf16*>(canon_lo.p);
     float* cb = static_cast<float*>(canon_b.p);
@@ -534,8 +647,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
         for (int j = 0; j < lp.w / 64; ++j)
           for (int r = 0; r < 64; ++r) idx.push_back(blk * D + hk[j] * 64 + r);
       ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
-      ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, int(idx.size()), lp.qkv_w, s));
-      if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, int(idx.size()), lp.qkv_w_lo, s));
+      const VitEmbed& em = h->modes[m].emb;
+      if (em.pruned) {  // input columns: the kept embedding channels
+        ELASTO_CUDA_TRY(gather2d_bf16(cw, D, di, int(idx.size()), eix(m), em.d_pad, lp.qkv_w, s));
+        if (split) ELASTO_CUDA_TRY(gather2d_bf16(cwl, D, di, int(idx.size()), eix(m), em.d_pad, lp.qkv_w_lo, s));
+      } else {
+        ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, int(idx.size()), lp.qkv_w, s));
+        if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, int(idx.size()), lp.qkv_w_lo, s));
+      }
       ELASTO_CUDA_TRY(gather_f32(cb, di, int(idx.size()), lp.qkv_b, s));
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
@@ -561,8 +680,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       for (int j = 0; j < lp.w / 64; ++j)
         for (int r = 0; r < 64; ++r) idx.push_back(hk[j] * 64 + r);
       ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
-      ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, D, di, int(idx.size()), lp.proj_w, s));
-      if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, D, di, int(idx.size()), lp.proj_w_lo, s));
+      const VitEmbed& em = h->modes[m].emb;
+      if (em.pruned) {  // output rows: the kept embedding channels
+        ELASTO_CUDA_TRY(gather2d_bf16(cw, D, eix(m), em.d_pad, di, int(idx.size()), lp.proj_w, s));
+        if (split) ELASTO_CUDA_TRY(gather2d_bf16(cwl, D, eix(m), em.d_pad, di, int(idx.size()), lp.proj_w_lo, s));
+      } else {
+        ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, D, di, int(idx.size()), lp.proj_w, s));
+        if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, D, di, int(idx.size()), lp.proj_w_lo, s));
+      }
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
     // fc1: rows F (padding rows stay zero), b1 entries F
@@ -582,8 +707,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       size_t fo = 0;
       for (int k = 0; k < l; ++k) fo += modes[m].n_mlp_kept[k];
       ELASTO_CUDA_TRY(cudaMemcpy(di, modes[m].mlp_kept + fo, size_t(lp.f) * 4, cudaMemcpyHostToDevice));
-      ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, lp.f, lp.fc1_w, s));
-      if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, lp.f, lp.fc1_w_lo, s));
+      const VitEmbed& em = h->modes[m].emb;
+      if (em.pruned) {  // input columns: the kept embedding channels
+        ELASTO_CUDA_TRY(gather2d_bf16(cw, D, di, lp.f, eix(m), em.d_pad, lp.fc1_w, s));
+        if (split) ELASTO_CUDA_TRY(gather2d_bf16(cwl, D, di, lp.f, eix(m), em.d_pad, lp.fc1_w_lo, s));
+      } else {
+        ELASTO_CUDA_TRY(gather_rows_bf16(cw, D, di, lp.f, lp.fc1_w, s));
+        if (split) ELASTO_CUDA_TRY(gather_rows_bf16(cwl, D, di, lp.f, lp.fc1_w_lo, s));
+      }
       ELASTO_CUDA_TRY(gather_f32(cb, di, lp.f, lp.fc1_b, s));
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
@@ -604,8 +735,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       idx.assign(modes[m].mlp_kept + fo, modes[m].mlp_kept + fo + lp.f);
       for (int k = lp.f; k < lp.f_pad; ++k) idx.push_back(-1);
       ELASTO_CUDA_TRY(cudaMemcpy(di, idx.data(), idx.size() * 4, cudaMemcpyHostToDevice));
-      ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, F, di, lp.f_pad, lp.fc2_w, s));
-      if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, F, di, lp.f_pad, lp.fc2_w_lo, s));
+      const VitEmbed& em = h->modes[m].emb;
+      if (em.pruned) {  // output rows: the kept embedding channels
+        ELASTO_CUDA_TRY(gather2d_bf16(cw, F, eix(m), em.d_pad, di, lp.f_pad, lp.fc2_w, s));
+        if (split) ELASTO_CUDA_TRY(gather2d_bf16(cwl, F, eix(m), em.d_pad, di, lp.f_pad, lp.fc2_w_lo, s));
+      } else {
+        ELASTO_CUDA_TRY(gather_cols_bf16(cw, D, F, di, lp.f_pad, lp.fc2_w, s));
+        if (split) ELASTO_CUDA_TRY(gather_cols_bf16(cwl, D, F, di, lp.f_pad, lp.fc2_w_lo, s));
+      }
       ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
     }
   }
@@ -640,19 +777,35 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   });
   if (st != ELASTO_OK) return st;
   ELASTO_CUDA_TRY(cudaDeviceSynchronize());
-  const int64_t lin_patch = int64_t(np) * D * kpe + int64_t(D) * C;
   for (int m = 0; m < n_modes; ++m) {
     VitMode& vm = h->modes[m];
-    vm.macs = lin_patch;
+    VitEmbed& em = vm.emb;
+    const int Dm = em.d_pad, dm = em.d;  // padded and kept embedding width
+    vm.macs = int64_t(np) * dm * kpe + int64_t(dm) * C;
     vm.launches = 3;  // patchify, patch GEMM, head
+    if (em.pruned) {
+      // patch rows [B * np, kpe] -> X rows past each class token, + position
+      // embedding (the class-token rows are written by the patchify kernel)
+      em.patch.n = h->n_plan_rows;
+      for (int i = 0; i < em.patch.n; ++i) {
+        em.patch.rows[i] = h->plan_rows[i] / n * np;
+        GemmPlan& gp = em.patch.plan[i];
+        st = gemm_plan(&gp, h->P, Bm * np, em.patch_w, Dm, kpe, em.patch_b, h->X, Dm, EPI_PATCH_POS_F32, h->status,
+                       em.patch_w_lo, em.patch.rows[i]);
+        if (st != ELASTO_OK) return st;
+        gp.args.patches = np;
+        gp.args.tokens = n;
+        gp.args.pos = em.pos;
+      }
+    }
     for (int l = 0; l < L; ++l) {
       VitLayerPack& lp = vm.layers[l];
-      vm.macs += int64_t(n) * D * 3 * lp.w + 2 * int64_t(n) * n * lp.w + int64_t(n) * lp.w * D +
-                 2 * int64_t(n) * D * lp.f;
+      vm.macs += int64_t(n) * dm * 3 * lp.w + 2 * int64_t(n) * n * lp.w + int64_t(n) * lp.w * dm +
+                 2 * int64_t(n) * dm * lp.f;
       vm.launches += 2;  // two LayerNorms
       if (lp.w > 0) {
         st = plan_set(lp.qkv, [&](GemmPlan& gp, int rows) {
-          return gemm_plan(&gp, h->Y, Mcap, lp.qkv_w, 3 * lp.w, D, lp.qkv_b, h->QKV, 3 * lp.w, EPI_BIAS_BF16,
+          return gemm_plan(&gp, h->Y, Mcap, lp.qkv_w, 3 * lp.w, Dm, lp.qkv_b, h->QKV, 3 * lp.w, EPI_BIAS_BF16,
                            h->status, lp.qkv_w_lo, rows);
         });
         if (st != ELASTO_OK) return st;
@@ -661,20 +814,20 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
         vm.launches += 2;
       }
       st = plan_set(lp.proj, [&](GemmPlan& gp, int rows) {
-        return gemm_plan(&gp, h->O, Mcap, lp.proj_w, D, lp.w, h->proj_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
+        return gemm_plan(&gp, h->O, Mcap, lp.proj_w, Dm, lp.w, em.proj_b[l], h->X, Dm, EPI_BIAS_RESID_F32, h->status,
                          lp.proj_w_lo, rows, lp.ld_proj);
       });
       if (st != ELASTO_OK) return st;
       if (lp.f > 0) {
         st = plan_set(lp.fc1, [&](GemmPlan& gp, int rows) {
-          return gemm_plan(&gp, h->Y, Mcap, lp.fc1_w, lp.f_pad, D, lp.fc1_b, h->H, lp.f_pad, EPI_BIAS_GELU_BF16,
+          return gemm_plan(&gp, h->Y, Mcap, lp.fc1_w, lp.f_pad, Dm, lp.fc1_b, h->H, lp.f_pad, EPI_BIAS_GELU_BF16,
                            h->status, lp.fc1_w_lo, rows);
         });
         if (st != ELASTO_OK) return st;
         vm.launches += 1;
       }
       st = plan_set(lp.fc2, [&](GemmPlan& gp, int rows) {
-        return gemm_plan(&gp, h->H, Mcap, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], h->X, D, EPI_BIAS_RESID_F32, h->status,
+        return gemm_plan(&gp, h->H, Mcap, lp.fc2_w, Dm, lp.f_pad, em.fc2_b[l], h->X, Dm, EPI_BIAS_RESID_F32, h->status,
                          lp.fc2_w_lo, rows, lp.ld_fc2);
       });
       if (st != ELASTO_OK) return st;
@@ -716,30 +869,40 @@ elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int b
   const VitMode& vm = h->modes[h->cur.load(std::memory_order_acquire)];
   const int n = h->n, D = d.dim, M = batch * n, Mp = batch * h->np, C = d.classes;
   const double img_elt = d.weight_dtype == ELASTO_BF16 ? 2 : 4;
+  const VitEmbed& em = vm.emb;
+  const int Dm = em.d_pad;  // residual-stream width (kept embedding channels, zero-padded)
   h->prof.begin();
-  ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, M, h->kpe, 0, 0, double(Mp) * h->kpe * img_elt + double(M) * h->kpe * 2),
-                patch_rows_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, s));
-  ELASTO_LAUNCH(gemm_rec(-1, M, D, h->kpe, 4, true), gemm_launch(h->patch.pick(M), M, s));
-  const double ln_bytes = double(M) * D * (4 + 2);
+  if (em.pruned) {
+    ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, Mp, h->kpe, 0, 0, double(Mp) * h->kpe * (img_elt + 2)),
+                  patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, h->X, em.cls,
+                                  em.pos, Dm, s));
+    ELASTO_LAUNCH(gemm_rec(-1, Mp, Dm, h->kpe, 4, false), gemm_launch(em.patch.pick(Mp), Mp, s));
+  } else {
+    ELASTO_LAUNCH(
+        make_rec(ELASTO_K_PATCHIFY, -1, M, h->kpe, 0, 0, double(Mp) * h->kpe * img_elt + double(M) * h->kpe * 2),
+        patch_rows_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, s));
+    ELASTO_LAUNCH(gemm_rec(-1, M, D, h->kpe, 4, true), gemm_launch(h->patch.pick(M), M, s));
+  }
+  const double ln_bytes = double(M) * Dm * (4 + 2);
   for (int l = 0; l < d.layers; ++l) {
     const VitLayerPack& lp = vm.layers[l];
-    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, D, 0, 0, ln_bytes),
-                  layernorm_launch(h->X, h->ln1_w[l], h->ln1_b[l], h->Y, M, D, s));
+    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, Dm, 0, 0, ln_bytes),
+                  layernorm_launch(h->X, em.ln1_w[l], em.ln1_b[l], h->Y, M, Dm, em.d, s));
     if (lp.w > 0) {
-      ELASTO_LAUNCH(gemm_rec(l, M, 3 * lp.w, D, 2, false), gemm_launch(lp.qkv.pick(M), M, s));
+      ELASTO_LAUNCH(gemm_rec(l, M, 3 * lp.w, Dm, 2, false), gemm_launch(lp.qkv.pick(M), M, s));
       ELASTO_LAUNCH(make_rec(ELASTO_K_ATTENTION, l, M, lp.w, n, 2.0 * batch * n * n * lp.w,
                              double(M) * lp.w * 2 * 4),
                     attn_launch(lp.attn, batch, s));
     }
-    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.w, 4, true), gemm_launch(lp.proj.pick(M), M, s));
-    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, D, 0, 0, ln_bytes),
-                  layernorm_launch(h->X, h->ln2_w[l], h->ln2_b[l], h->Y, M, D, s));
-    if (lp.f > 0) ELASTO_LAUNCH(gemm_rec(l, M, lp.f_pad, D, 2, false), gemm_launch(lp.fc1.pick(M), M, s));
-    ELASTO_LAUNCH(gemm_rec(l, M, D, lp.f_pad, 4, true), gemm_launch(lp.fc2.pick(M), M, s));
+    ELASTO_LAUNCH(gemm_rec(l, M, Dm, lp.w, 4, true), gemm_launch(lp.proj.pick(M), M, s));
+    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, Dm, 0, 0, ln_bytes),
+                  layernorm_launch(h->X, em.ln2_w[l], em.ln2_b[l], h->Y, M, Dm, em.d, s));
+    if (lp.f > 0) ELASTO_LAUNCH(gemm_rec(l, M, lp.f_pad, Dm, 2, false), gemm_launch(lp.fc1.pick(M), M, s));
+    ELASTO_LAUNCH(gemm_rec(l, M, Dm, lp.f_pad, 4, true), gemm_launch(lp.fc2.pick(M), M, s));
   }
-  ELASTO_LAUNCH(make_rec(ELASTO_K_HEAD, -1, batch, C, D, double(batch) * C * D,
-                         double(batch) * D * 4 + double(C) * D * 4 + double(batch) * C * 4),
-                head_launch(h->X, batch, n, D, h->norm_w, h->norm_b, h->head_w, h->head_b, C, logits, s));
+  ELASTO_LAUNCH(make_rec(ELASTO_K_HEAD, -1, batch, C, Dm, double(batch) * C * em.d,
+                         double(batch) * Dm * 4 + double(C) * Dm * 4 + double(batch) * C * 4),
+                head_launch(h->X, batch, n, Dm, em.d, em.norm_w, em.norm_b, em.head_w, h->head_b, C, logits, s));
   return ELASTO_OK;
 }
 
@@ -1019,7 +1182,8 @@ elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int wh
     return ELASTO_ERR_INVALID_ARG;
   }
   const VitLayerPack& lp = h->modes[mode].layers[layer];
-  const size_t D = h->d.dim;
+  const VitEmbed& em = h->modes[mode].emb;
+  const size_t D = em.d, Dm = em.d_pad;  // kept embedding width; stored rows have Dm entries
   size_t need = 0;
   const void* src = nullptr;
   switch (which) {
@@ -1071,9 +1235,13 @@ elasto_status elasto_debug_export_packed(elasto_t h, int mode, int layer, int wh
     return ELASTO_OK;
   }
   if (which == 5) {
-    // stored [d, f_pad]; export [d, f]
+    // stored [d_pad, f_pad]; export [d, f]
     ELASTO_CUDA_TRY(cudaMemcpy2D(host_dst, size_t(lp.f) * 2, src, size_t(lp.f_pad) * 2, size_t(lp.f) * 2, D,
                                  cudaMemcpyDeviceToHost));
+  } else if (which == 0 || which == 3) {
+    // stored [rows, d_pad]; export [rows, d]
+    const size_t rows = which == 0 ? size_t(3) * lp.w : size_t(lp.f);
+    ELASTO_CUDA_TRY(cudaMemcpy2D(host_dst, D * 2, src, Dm * 2, D * 2, rows, cudaMemcpyDeviceToHost));
   } else {
     ELASTO_CUDA_TRY(cudaMemcpy(host_dst, src, need, cudaMemcpyDeviceToHost));
   }

@@ -180,7 +180,10 @@ cudaError_t attn_launch(const AttnPlan& p, int batch, cudaStream_t s);
 cudaError_t attn_init_attributes();
 
 // ---------------------------------------------------------------- small kernels
-cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf16* y, int rows, int d,
+// y [rows, d] bf16 = LayerNorm of x [rows, d] fp32 (eps 1e-6) with statistics
+// over the first d_true channels; channels [d_true, d) of x must be zero and
+// of g, b zero (the padding of a pruned embedding width). d % 64 == 0, d <= 1024.
+cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf16* y, int rows, int d, int d_true,
                              cudaStream_t s);
 cudaError_t softmax_launch(const float* x, float* y, int rows, int cols, cudaStream_t s);
 // images [B, H, W, C] (bf16 or fp32) -> A [B * np, P*P*C] bf16 in (ky, kx, c)
@@ -196,14 +199,20 @@ cudaError_t patch_rows_launch(const void* images, int img_dtype, int B, int H, i
 // over the batch: row 0 of an image = cls + pos[0], row t >= 1 = pos[t] + b_pe.
 cudaError_t token_addend_launch(const float* cls, const float* pos, const float* patch_b, int n, int d, int B,
                                 float* dst, cudaStream_t s);
-// logits[b, c] = LN(X[b * n, :]) . head_w[c, :] + head_b[c], all fp32.
-cudaError_t head_launch(const float* X, int B, int n, int d, const float* g, const float* b, const float* Wh,
+// logits[b, c] = LN(X[b * n, :]) . head_w[c, :] + head_b[c], all fp32; rows of
+// width d, LayerNorm statistics over the first d_true channels (the rest zero).
+cudaError_t head_launch(const float* X, int B, int n, int d, int d_true, const float* g, const float* b, const float* Wh,
                         const float* bh, int C, float* logits, cudaStream_t s);
 // gathers for create-time packing
 cudaError_t gather_rows_bf16(const bf16* src, int cols, const int32_t* idx, int nidx, bf16* dst, cudaStream_t s);
 cudaError_t gather_cols_bf16(const bf16* src, int rows, int cols, const int32_t* idx, int nidx, bf16* dst,
                              cudaStream_t s);
-cudaError_t gather_f32(const float* src, const int32_t* idx, int nidx, float* dst, cudaStream_t s);
+cudaError_t gather_f32(const float* src, const int32_t* idx, int nidx, float* dst, cudaStream_t s);  // -1: zero
+// dst [nr, nc] = src[ri, ci] of a row-major source with src_cols columns; -1 in ri or ci gives zero.
+cudaError_t gather2d_bf16(const bf16* src, int src_cols, const int32_t* ri, int nr, const int32_t* ci, int nc, bf16* dst,
+                          cudaStream_t s);
+cudaError_t gather2d_f32(const float* src, int src_cols, const int32_t* ri, int nr, const int32_t* ci, int nc,
+                         float* dst, cudaStream_t s);
 cudaError_t convert_to_bf16(const void* src, int src_dtype, size_t n, bf16* dst, cudaStream_t s);
 // dst = bf16(x - bf16(x)) for fp32 sources (the low plane of a bf16 pair); zeros for bf16 sources.
 cudaError_t convert_to_bf16_lo(const void* src, int src_dtype, size_t n, bf16* dst, cudaStream_t s);

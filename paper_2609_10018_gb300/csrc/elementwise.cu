@@ -114,11 +114,15 @@ __device__ __forceinline__ float warp_max(float v) {
   return v;
 }
 
-// One warp per row; each lane holds VEC float2 pairs (d = 64 * VEC).
+// One warp per row; each lane holds VEC float2 pairs (row width 64 * VEC).
+// The statistics are over the first d_true channels: the remaining `pad`
+// channels hold zeros (an embedding-pruned width padded to 64), so they add
+// nothing to the sum and pad * mean^2 to the centred sum of squares, which is
+// taken back out. gamma and beta are zero there, so y is zero there too.
 template <int VEC>
 __global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict__ x, const float* __restrict__ g,
                                                         const float* __restrict__ b, bf16* __restrict__ y,
-                                                        int rows, float inv_d) {
+                                                        int rows, float inv_d, float pad) {
   pdl_wait();
   pdl_trigger();
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
@@ -140,7 +144,7 @@ __global__ void __launch_bounds__(256) layernorm_kernel(const float* __restrict_
     const float a = v[i].x - mean, c = v[i].y - mean;
     ss += a * a + c * c;
   }
-  const float rstd = rsqrtf(warp_sum(ss) * inv_d + 1e-6f);
+  const float rstd = rsqrtf((warp_sum(ss) - pad * mean * mean) * inv_d + 1e-6f);
   const float2* g2 = reinterpret_cast<const float2*>(g);
   const float2* b2 = reinterpret_cast<const float2*>(b);
   uint32_t* yr = reinterpret_cast<uint32_t*>(y + static_cast<size_t>(row) * D);
@@ -170,16 +174,17 @@ __global__ void __launch_bounds__(256) softmax_kernel(const float* __restrict__ 
 
 }  // namespace
 
-cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf16* y, int rows, int d,
+cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf16* y, int rows, int d, int d_true,
                              cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
+  if (d % 64 != 0 || d_true <= 0 || d_true > d) return cudaErrorInvalidValue;
   const dim3 grid((rows + 7) / 8);
-  const float inv_d = 1.0f / static_cast<float>(d);
+  const float inv_d = 1.0f / static_cast<float>(d_true), pad = static_cast<float>(d - d_true);
   switch (d / 64) {
 #define LN_CASE(V) \
-  case V: return launch_pdl(layernorm_kernel<V>, grid, dim3(256), 0, s, x, g, b, y, rows, inv_d);
-    LN_CASE(1) LN_CASE(2) LN_CASE(3) LN_CASE(4) LN_CASE(5) LN_CASE(6) LN_CASE(8) LN_CASE(10) LN_CASE(12)
-    LN_CASE(16)
+  case V: return launch_pdl(layernorm_kernel<V>, grid, dim3(256), 0, s, x, g, b, y, rows, inv_d, pad);
+    LN_CASE(1) LN_CASE(2) LN_CASE(3) LN_CASE(4) LN_CASE(5) LN_CASE(6) LN_CASE(7) LN_CASE(8) LN_CASE(9)
+    LN_CASE(10) LN_CASE(11) LN_CASE(12) LN_CASE(13) LN_CASE(14) LN_CASE(15) LN_CASE(16)
 #undef LN_CASE
     default: return cudaErrorInvalidValue;
   }
@@ -345,7 +350,9 @@ constexpr int HEAD_CLASSES = 16;  // classes per CTA (two per warp)
 // tokens into shared memory (fp32), then each warp computes 2 classes x 8
 // images of dot products. The classifier row's loads are issued 4 float4 at a
 // time, so a warp has several HBM/L2 requests in flight instead of one.
-__global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, int B, int n, int d,
+// d is the row width of X and Wh; the LayerNorm statistics cover the first
+// d_true channels (the rest are the zero padding of a pruned width).
+__global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, int B, int n, int d, int d_true,
                                                    const float* __restrict__ g, const float* __restrict__ bta,
                                                    const float* __restrict__ Wh, const float* __restrict__ bh, int C,
                                                    float* __restrict__ logits) {
@@ -358,15 +365,15 @@ __global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, 
   if (warp < nimg) {
     const float* xr = X + static_cast<size_t>(b0 + warp) * n * d;  // class token row
     float s = 0.0f;
-    for (int c = lane; c < d; c += 32) s += xr[c];
-    const float mean = warp_sum(s) / d;
+    for (int c = lane; c < d_true; c += 32) s += xr[c];
+    const float mean = warp_sum(s) / d_true;
     float ss = 0.0f;
-    for (int c = lane; c < d; c += 32) {
+    for (int c = lane; c < d_true; c += 32) {
       const float a = xr[c] - mean;
       ss += a * a;
     }
-    const float rstd = rsqrtf(warp_sum(ss) / d + 1e-6f);
-    for (int c = lane; c < d; c += 32) sy[warp * d + c] = (xr[c] - mean) * rstd * g[c] + bta[c];
+    const float rstd = rsqrtf(warp_sum(ss) / d_true + 1e-6f);
+    for (int c = lane; c < d; c += 32) sy[warp * d + c] = c < d_true ? (xr[c] - mean) * rstd * g[c] + bta[c] : 0.0f;
   }
   __syncthreads();
   const int c0 = blockIdx.y * HEAD_CLASSES;
@@ -398,12 +405,13 @@ __global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, 
 
 }  // namespace
 
-cudaError_t head_launch(const float* X, int B, int n, int d, const float* g, const float* b, const float* Wh,
-                        const float* bh, int C, float* logits, cudaStream_t s) {
+cudaError_t head_launch(const float* X, int B, int n, int d, int d_true, const float* g, const float* b,
+                        const float* Wh, const float* bh, int C, float* logits, cudaStream_t s) {
   if (B <= 0) return cudaSuccess;
+  if (d % 4 != 0 || d_true <= 0 || d_true > d) return cudaErrorInvalidValue;
   dim3 grid((B + HEAD_IMGS - 1) / HEAD_IMGS, (C + HEAD_CLASSES - 1) / HEAD_CLASSES);
-  return launch_pdl(head_kernel, grid, dim3(256), HEAD_IMGS * d * sizeof(float), s, X, B, n, d, g, b, Wh, bh, C,
-                    logits);
+  return launch_pdl(head_kernel, grid, dim3(256), HEAD_IMGS * d * sizeof(float), s, X, B, n, d, d_true, g, b, Wh, bh,
+                    C, logits);
 }
 
 // ---------------------------------------------------------------- packing
@@ -433,7 +441,20 @@ __global__ void gather_cols_kernel(const bf16* __restrict__ src, int rows, int c
 __global__ void gather_f32_kernel(const float* __restrict__ src, const int32_t* __restrict__ idx, int nidx,
                                   float* __restrict__ dst) {
   const int t = blockIdx.x * blockDim.x + threadIdx.x;
-  if (t < nidx) dst[t] = src[idx[t]];
+  if (t < nidx) dst[t] = idx[t] >= 0 ? src[idx[t]] : 0.0f;
+}
+
+// dst [nr, nc] = src [ri, ci] (src row-major with src_cols columns); an index
+// of -1 in either list gives a zero (padding rows or columns).
+template <typename T>
+__global__ void gather2d_kernel(const T* __restrict__ src, int src_cols, const int32_t* __restrict__ ri, int nr,
+                                const int32_t* __restrict__ ci, int nc, T* __restrict__ dst) {
+  const size_t total = static_cast<size_t>(nr) * nc;
+  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
+       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const int r = ri[t / nc], c = ci[t % nc];
+    dst[t] = (r >= 0 && c >= 0) ? src[static_cast<size_t>(r) * src_cols + c] : T(0.0f);
+  }
 }
 
 template <typename T>
@@ -474,6 +495,18 @@ cudaError_t gather_cols_bf16(const bf16* src, int rows, int cols, const int32_t*
                              cudaStream_t s) {
   if (nidx <= 0 || rows <= 0) return cudaSuccess;
   gather_cols_kernel<<<grid_for(static_cast<size_t>(rows) * nidx), 256, 0, s>>>(src, rows, cols, idx, nidx, dst);
+  return cudaGetLastError();
+}
+cudaError_t gather2d_bf16(const bf16* src, int src_cols, const int32_t* ri, int nr, const int32_t* ci, int nc, bf16* dst,
+                          cudaStream_t s) {
+  if (nr <= 0 || nc <= 0) return cudaSuccess;
+  gather2d_kernel<bf16><<<grid_for(static_cast<size_t>(nr) * nc), 256, 0, s>>>(src, src_cols, ri, nr, ci, nc, dst);
+  return cudaGetLastError();
+}
+cudaError_t gather2d_f32(const float* src, int src_cols, const int32_t* ri, int nr, const int32_t* ci, int nc,
+                         float* dst, cudaStream_t s) {
+  if (nr <= 0 || nc <= 0) return cudaSuccess;
+  gather2d_kernel<float><<<grid_for(static_cast<size_t>(nr) * nc), 256, 0, s>>>(src, src_cols, ri, nr, ci, nc, dst);
   return cudaGetLastError();
 }
 cudaError_t gather_f32(const float* src, const int32_t* idx, int nidx, float* dst, cudaStream_t s) {

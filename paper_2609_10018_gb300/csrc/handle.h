@@ -27,8 +27,24 @@ struct VitLayerPack {
   AttnPlan attn;
 };
 
+// The parameters that carry the embedding width. A mode that keeps every
+// channel points at the handle's copies; an embedding-pruned mode (Section
+// 4.1) has its own, holding the kept channels E first and zero padding up to
+// d_pad (a multiple of 64), so the residual stream X is [rows, d_pad] with
+// zeros past d.
+struct VitEmbed {
+  int d = 0, d_pad = 0;  // kept channels, padded width
+  bool pruned = false;
+  bf16 *patch_w = nullptr, *patch_w_lo = nullptr;  // [d_pad, P*P*C]
+  float *patch_b = nullptr, *cls = nullptr, *pos = nullptr;  // [d_pad], [d_pad], [n, d_pad]
+  std::vector<float*> ln1_w, ln1_b, ln2_w, ln2_b, proj_b, fc2_b;  // per layer, [d_pad]
+  float *norm_w = nullptr, *norm_b = nullptr, *head_w = nullptr;  // [d_pad], [d_pad], [C, d_pad]
+  GemmPlanSet patch;  // pruned modes: patch rows -> X past the class token, + position embedding
+};
+
 struct VitMode {
   std::vector<VitLayerPack> layers;
+  VitEmbed emb;
   size_t packed_bytes = 0;  // bytes of packed weights this mode reads
   int64_t macs = 0;
   int launches = 0;

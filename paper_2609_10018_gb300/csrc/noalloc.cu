@@ -126,21 +126,22 @@ extern "C" elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const 
   bf16* H = reinterpret_cast<bf16*>(S + L.H);
   bf16* P = reinterpret_cast<bf16*>(S + L.P);
 
-  const int n = h->n, D = d.dim, M = batch * n, Mp = batch * h->np;
+  const VitEmbed& em = vm.emb;
+  const int n = h->n, D = em.d_pad, M = batch * n, Mp = batch * h->np;  // D: residual-stream width of this mode
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   GemmPlan gp;
-  st = gemm_plan(&gp, P, Mp, h->patch_w, D, h->kpe, h->patch_b, X, D, EPI_PATCH_POS_F32, h->status,
-                 h->patch_w_lo);
+  st = gemm_plan(&gp, P, Mp, em.patch_w, D, h->kpe, em.patch_b, X, D, EPI_PATCH_POS_F32, h->status,
+                 em.patch_w_lo);
   if (st != ELASTO_OK) return st;
   gp.args.patches = h->np;
   gp.args.tokens = n;
-  gp.args.pos = h->pos;
+  gp.args.pos = em.pos;
   ELASTO_CUDA_TRY(
-      patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, P, X, h->cls, h->pos, D, s));
+      patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, P, X, em.cls, em.pos, D, s));
   ELASTO_CUDA_TRY(gemm_launch(gp, Mp, s));
   for (int l = 0; l < d.layers; ++l) {
     const VitLayerPack& lp = vm.layers[l];
-    ELASTO_CUDA_TRY(layernorm_launch(X, h->ln1_w[l], h->ln1_b[l], Y, M, D, s));
+    ELASTO_CUDA_TRY(layernorm_launch(X, em.ln1_w[l], em.ln1_b[l], Y, M, D, em.d, s));
     if (lp.w > 0) {
       GemmPlan qkv;
       AttnPlan at;
@@ -152,11 +153,11 @@ extern "C" elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const 
       ELASTO_CUDA_TRY(attn_launch(at, batch, s));
     }
     GemmPlan proj, fc2;
-    if ((st = gemm_plan(&proj, O, M, lp.proj_w, D, lp.w, h->proj_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
+    if ((st = gemm_plan(&proj, O, M, lp.proj_w, D, lp.w, em.proj_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
                         lp.proj_w_lo, 0, lp.ld_proj)) != ELASTO_OK)
       return st;
     ELASTO_CUDA_TRY(gemm_launch(proj, M, s));
-    ELASTO_CUDA_TRY(layernorm_launch(X, h->ln2_w[l], h->ln2_b[l], Y, M, D, s));
+    ELASTO_CUDA_TRY(layernorm_launch(X, em.ln2_w[l], em.ln2_b[l], Y, M, D, em.d, s));
     if (lp.f > 0) {
       GemmPlan fc1;
       if ((st = gemm_plan(&fc1, Y, M, lp.fc1_w, lp.f_pad, D, lp.fc1_b, H, lp.f_pad, EPI_BIAS_GELU_BF16,
@@ -164,11 +165,12 @@ extern "C" elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const 
         return st;
       ELASTO_CUDA_TRY(gemm_launch(fc1, M, s));
     }
-    if ((st = gemm_plan(&fc2, H, M, lp.fc2_w, D, lp.f_pad, h->fc2_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
+    if ((st = gemm_plan(&fc2, H, M, lp.fc2_w, D, lp.f_pad, em.fc2_b[l], X, D, EPI_BIAS_RESID_F32, h->status,
                         lp.fc2_w_lo, 0, lp.ld_fc2)) != ELASTO_OK)
       return st;
     ELASTO_CUDA_TRY(gemm_launch(fc2, M, s));
   }
-  ELASTO_CUDA_TRY(head_launch(X, batch, n, D, h->norm_w, h->norm_b, h->head_w, h->head_b, d.classes, logits, s));
+  ELASTO_CUDA_TRY(
+      head_launch(X, batch, n, D, em.d, em.norm_w, em.norm_b, em.head_w, h->head_b, d.classes, logits, s));
   return ELASTO_OK;
 }

@@ -59,7 +59,8 @@ elasto_status elasto_op_layernorm(void* stream, const float* x, const float* gam
     set_error("elasto_op_layernorm: d must be 64 x {1..6, 8, 10, 12, 16}");
     return ELASTO_ERR_UNSUPPORTED;
   }
-  ELASTO_CUDA_TRY(layernorm_launch(x, gamma, beta, static_cast<bf16*>(y), rows, d, static_cast<cudaStream_t>(stream)));
+  ELASTO_CUDA_TRY(
+      layernorm_launch(x, gamma, beta, static_cast<bf16*>(y), rows, d, d, static_cast<cudaStream_t>(stream)));
   return ELASTO_OK;
 }
 

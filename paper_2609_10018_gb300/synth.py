@@ -191,6 +191,20 @@ def make_vit_tables(cfg: VitConfig, seed: int | None = None,
     return modes
 
 
+def with_embedding(cfg: VitConfig, tables, widths, seed: int | None = None):
+    """Copies of the mode tables that also prune the embedding width: mode m
+    keeps widths[m] of the d channels (None: all), nested across the modes
+    (one seeded permutation, each mode the sorted first widths[m] entries)."""
+    rng = np.random.default_rng([cfg.seeds[1] if seed is None else seed, 1_000_003])
+    perm = rng.permutation(cfg.dim)
+    out = []
+    for t, k in zip(tables, widths):
+        t = dict(t)
+        t["embed"] = None if k is None else np.sort(perm[:k]).astype(np.int32)
+        out.append(t)
+    return out
+
+
 def make_images(cfg, batch: int, seed: int | None = None) -> np.ndarray:
     """[B, H, W, C] pixels U[0, 1) (no normalisation), stored in cfg.dtype."""
     rng = np.random.default_rng(cfg.seeds[2] if seed is None else seed)

@@ -73,6 +73,9 @@ def _create(lib, desc, ws, mt, n):
     (lambda t: t[1]["heads"].__setitem__(0, np.array([0, 3], np.int32)), binding.ERR_BAD_TABLE),     # out of range
     (lambda t: t[1]["mlp"].__setitem__(2, np.array([-1, 5], np.int32)), binding.ERR_BAD_TABLE),      # negative
     (lambda t: t[1]["heads"].__setitem__(0, np.arange(4, dtype=np.int32)), binding.ERR_BAD_TABLE),   # too many
+    (lambda t: t[1].__setitem__("embed", np.array([3, 2, 9], np.int32)), binding.ERR_BAD_TABLE),     # embed unsorted
+    (lambda t: t[1].__setitem__("embed", np.array([0, 192], np.int32)), binding.ERR_BAD_TABLE),      # embed >= dim
+    (lambda t: t[1].__setitem__("embed", np.arange(193, dtype=np.int32) % 192), binding.ERR_BAD_TABLE),  # > dim
 ])
 def test_bad_tables_rejected_before_cuda(lib, mutate, code):
     tables = synth.make_vit_tables(synth.TINY)
