@@ -368,11 +368,66 @@ def main():
         line["cpu_baseline"] = oracle_cpu_baseline(cfg)
     model.close()
     if rank == 0 and not args.quick:
+        line["embed_ladder"] = embed_ladder(torch, binding, synth, weights, images, peaks)
         line["resnet50"] = resnet50_section(torch, binding, synth, peaks)
     if rank == 0:
         print(json.dumps(line))
     if dist:
         dist.destroy_process_group()
+
+
+# Table 1 (Section 6.1), compression ratio 0.40: FLOPs (G) of the Level-1 ... Level-6 DNs of ViT-B
+TABLE1_CR040_GFLOPS = [5.70, 7.58, 9.57, 11.38, 13.99, 16.86]
+
+
+def embed_ladder(torch, binding, synth, weights, images, peaks, cr=0.4, rounds=5, steps=10, warmup=3):
+    """Six DNs that prune the embedding width d together with the heads and
+    the MLP channels (Section 4.1), on the compression ladder of Eq. 1:
+    p = 1 - (1 - CR)^(1/N) per round, so Level L keeps the fraction
+    (1 - CR)^((N + 1 - L) / N) of every width (nested kept sets, Eq. 8).
+    ViT-B at batch 256, images/s per level, with the MACs each level executes
+    next to the FLOPs Table 1 prints for CR = 0.40 (the paper's exact widths
+    are not given)."""
+    cfg = synth.VIT_B
+    B = images.shape[0]
+    rng = np.random.default_rng(cfg.seeds[1] + 17)
+    pd, ph, pf = rng.permutation(cfg.dim), rng.permutation(cfg.heads), rng.permutation(cfg.mlp)
+    tables, widths = [], []
+    for level in range(rounds + 1, 0, -1):  # mode 0 = Level-6 (full) ... mode 5 = Level-1 (core)
+        r = (1.0 - cr) ** ((rounds + 1 - level) / rounds)
+        dm, hm, fm = round(r * cfg.dim), max(1, round(r * cfg.heads)), round(r * cfg.mlp)
+        widths.append({"level": level, "d": dm, "heads": hm, "mlp": fm})
+        tables.append({"heads": [np.sort(ph[:hm]).astype(np.int32)] * cfg.layers,
+                       "mlp": [np.sort(pf[:fm]).astype(np.int32)] * cfg.layers,
+                       "embed": None if dm == cfg.dim else np.sort(pd[:dm]).astype(np.int32)})
+    model = binding.ElasticModel.vit(cfg, weights, tables, max_batch=B)
+    logits = torch.empty(B, cfg.classes, dtype=torch.float32, device="cuda")
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    out = []
+    for m, wdt in enumerate(widths):
+        model.set_mode(m)
+        for _ in range(warmup):
+            model.forward(sh, images.data_ptr(), B, logits.data_ptr())
+        ts = []
+        for _ in range(steps):
+            flush.fill_(1.0)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            model.forward(sh, images.data_ptr(), B, logits.data_ptr())
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        macs = model.query(binding.Q_MODE_MACS, m)
+        ips = B * steps / (sum(ts) / 1e3)
+        out.append({**wdt, "images_per_s": ips, "gmac_per_image": macs / 1e9,
+                    "table1_gflops_cr040": TABLE1_CR040_GFLOPS[wdt["level"] - 1],
+                    "tflops": 2.0 * macs * ips / 1e12, "frac_of_bf16_peak": 2.0 * macs * ips / 1e12 / peaks["bf16_tflops"],
+                    "packed_weight_mb": model.query(binding.Q_PACKED_BYTES, m) / 1e6})
+    model.close()
+    return {"batch": B, "cr": cr, "rounds": rounds, "levels": out,
+            "note": "Table 1 counts FLOPs as multiply-accumulates of the linear layers; gmac_per_image adds attention"}
 
 
 def resnet50_section(torch, binding, synth, peaks, B=128, steps=20, warmup=3):
