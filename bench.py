@@ -145,6 +145,20 @@ def oracle_cpu_baseline(cfg, budget_s: float = 12.0, mode: int = 0):
                       f"({dt:.1f} s; numpy/OpenBLAS on {cores} host threads)"}
 
 
+def whole_job_rate(dist, local_ms: float, units_per_rank: int, world: int, device: str = "cuda"):
+    """The timed region of the slowest rank (ms, max over ranks) and the
+    whole-job throughput: the units all ranks processed / that time. Every
+    rank runs its own replica on its own batch (weak scaling, no exchange
+    between replicas), so the only collective is this one reduction."""
+    total_ms = float(local_ms)
+    if dist is not None and world > 1:
+        import torch
+        t = torch.tensor([total_ms], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    return total_ms, world * units_per_rank / (total_ms / 1e3)
+
+
 def run_reference(args):
     """Reference arm: the fp64 oracle on the host cores, same metric and
     workload, each step a bounded sample (1 image) of it."""
@@ -289,12 +303,7 @@ def main():
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    total_ms = float(sum(times))
-    if dist:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    value = world * B * args.steps / (total_ms / 1e3)
+    total_ms, value = whole_job_rate(dist, float(sum(times)), B * args.steps, world)
     macs_img = model.query(binding.Q_MODE_MACS, args.mode)
     tflops = 2.0 * macs_img * B * args.steps / (float(sum(times)) / 1e3) / 1e12
     launches = model.query(binding.Q_LAUNCHES, args.mode)
