@@ -338,8 +338,9 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       }
     }
   }
+  const int addend_rows = (1 + (128 + n - 1) / n) * n;
   struct EmbOff {
-    size_t patch_w = 0, patch_lo = 0, patch_b = 0, cls = 0, pos = 0, norm_w = 0, norm_b = 0, head_w = 0;
+    size_t patch_w = 0, patch_lo = 0, patch_b = 0, cls = 0, pos = 0, norm_w = 0, norm_b = 0, head_w = 0, addend = 0;
     std::vector<size_t> lvec;  // per layer: ln1_w, ln1_b, ln2_w, ln2_b, proj_b, fc2_b
   };
   std::vector<EmbOff> eoffs(n_modes);
@@ -358,6 +359,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       eo.norm_w = bump.take(size_t(Dm) * 4);
       eo.norm_b = bump.take(size_t(Dm) * 4);
       eo.head_w = bump.take(size_t(C) * Dm * 4);
+      eo.addend = bump.take(size_t(addend_rows) * Dm * 4);
       for (int k = 0; k < 6 * L; ++k) eo.lvec.push_back(bump.take(size_t(Dm) * 4));
     }
     size_t view = 0;
@@ -397,7 +399,10 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   const size_t o_X = bump.take(rows * D * 4), o_Y = bump.take(rows * D * 2);
   const size_t o_QKV = bump.take(rows * 3 * std::max(wmax, 64) * 2), o_O = bump.take(rows * std::max(wmax, 64) * 2);
   const size_t o_H = bump.take(rows * std::max(fmax, 8) * 2), o_P = bump.take(rows * kpe * 2);
-  const size_t o_tok = bump.take(rows * D * 4);  // per-token addend of the patch projection
+  // per-token addend of the patch projection: periodic in the token index, so
+  // k images' worth (k * n >= n + 128 rows) serve every batch
+  h->addend_rows = (1 + (128 + n - 1) / n) * n;
+  const size_t o_tok = bump.take(size_t(h->addend_rows) * D * 4);
   const size_t img_bytes = size_t(Bm) * d->img_h * d->img_w * d->img_c * dtype_size(d->weight_dtype);
   const size_t o_img = bump.take(img_bytes), o_logit = bump.take(size_t(Bm) * C * 4);
   const size_t o_status = bump.take(64);
@@ -467,6 +472,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     em.norm_w = reinterpret_cast<float*>(A + eo.norm_w);
     em.norm_b = reinterpret_cast<float*>(A + eo.norm_b);
     em.head_w = reinterpret_cast<float*>(A + eo.head_w);
+    em.addend = reinterpret_cast<float*>(A + eo.addend);
     for (int l = 0; l < L; ++l) {
       em.ln1_w.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 0]));
       em.ln1_b.push_back(reinterpret_cast<float*>(A + eo.lvec[6 * l + 1]));
@@ -754,7 +760,13 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   // Patch projection over token-ordered rows (class-token slots are zero
   // rows): X = addend + P W_pe^T, addend = cls + pos[0] on class tokens and
   // pos[t] + b_pe on patch tokens (Section 4.1: N = HW/P^2 patches, n = N + 1).
-  ELASTO_CUDA_TRY(token_addend_launch(h->cls, h->pos, h->patch_b, n, D, Bm, h->tok_addend, 0));
+  ELASTO_CUDA_TRY(token_addend_launch(h->cls, h->pos, h->patch_b, n, D, h->addend_rows / n, h->tok_addend, 0));
+  for (int m = 0; m < n_modes; ++m) {
+    const VitEmbed& em = h->modes[m].emb;
+    if (em.pruned)
+      ELASTO_CUDA_TRY(
+          token_addend_launch(em.cls, em.pos, em.patch_b, n, em.d_pad, h->addend_rows / n, em.addend, 0));
+  }
   // plan variants for 1, 8 and 32 images (those below max_batch) and max_batch
   h->n_plan_rows = 0;
   for (int b : {1, 8, 32})
@@ -773,7 +785,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   st = plan_set(h->patch, [&](GemmPlan& gp, int rows) {
     elasto_status r = gemm_plan(&gp, h->P, Mcap, h->patch_w, D, kpe, nullptr, h->X, D, EPI_BIAS_RESID_F32,
                                 h->status, h->patch_w_lo, rows);
-    return r != ELASTO_OK ? r : gemm_set_residual_source(&gp, h->tok_addend, Mcap);
+    return r != ELASTO_OK ? r : gemm_set_residual_source(&gp, h->tok_addend, h->addend_rows, n);
   });
   if (st != ELASTO_OK) return st;
   ELASTO_CUDA_TRY(cudaDeviceSynchronize());
@@ -783,20 +795,13 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     const int Dm = em.d_pad, dm = em.d;  // padded and kept embedding width
     vm.macs = int64_t(np) * dm * kpe + int64_t(dm) * C;
     vm.launches = 3;  // patchify, patch GEMM, head
-    if (em.pruned) {
-      // patch rows [B * np, kpe] -> X rows past each class token, + position
-      // embedding (the class-token rows are written by the patchify kernel)
-      em.patch.n = h->n_plan_rows;
-      for (int i = 0; i < em.patch.n; ++i) {
-        em.patch.rows[i] = h->plan_rows[i] / n * np;
-        GemmPlan& gp = em.patch.plan[i];
-        st = gemm_plan(&gp, h->P, Bm * np, em.patch_w, Dm, kpe, em.patch_b, h->X, Dm, EPI_PATCH_POS_F32, h->status,
-                       em.patch_w_lo, em.patch.rows[i]);
-        if (st != ELASTO_OK) return st;
-        gp.args.patches = np;
-        gp.args.tokens = n;
-        gp.args.pos = em.pos;
-      }
+    if (em.pruned) {  // the patch projection at this mode's width, its own addend
+      st = plan_set(em.patch, [&](GemmPlan& gp, int rows) {
+        elasto_status r = gemm_plan(&gp, h->P, Mcap, em.patch_w, Dm, kpe, nullptr, h->X, Dm, EPI_BIAS_RESID_F32,
+                                    h->status, em.patch_w_lo, rows);
+        return r != ELASTO_OK ? r : gemm_set_residual_source(&gp, em.addend, h->addend_rows, n);
+      });
+      if (st != ELASTO_OK) return st;
     }
     for (int l = 0; l < L; ++l) {
       VitLayerPack& lp = vm.layers[l];
@@ -872,17 +877,12 @@ elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int b
   const VitEmbed& em = vm.emb;
   const int Dm = em.d_pad;  // residual-stream width (kept embedding channels, zero-padded)
   h->prof.begin();
-  if (em.pruned) {
-    ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, Mp, h->kpe, 0, 0, double(Mp) * h->kpe * (img_elt + 2)),
-                  patchify_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, h->X, em.cls,
-                                  em.pos, Dm, s));
-    ELASTO_LAUNCH(gemm_rec(-1, Mp, Dm, h->kpe, 4, false), gemm_launch(em.patch.pick(Mp), Mp, s));
-  } else {
-    ELASTO_LAUNCH(
-        make_rec(ELASTO_K_PATCHIFY, -1, M, h->kpe, 0, 0, double(Mp) * h->kpe * img_elt + double(M) * h->kpe * 2),
-        patch_rows_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, s));
-    ELASTO_LAUNCH(gemm_rec(-1, M, D, h->kpe, 4, true), gemm_launch(h->patch.pick(M), M, s));
-  }
+  ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, M, h->kpe, 0, 0, double(Mp) * h->kpe * img_elt + double(M) * h->kpe * 2),
+                patch_rows_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, s));
+  // patch projection; the addend (class token / position embedding / b_pe)
+  // is periodic in the token and read from L2
+  ELASTO_LAUNCH(gemm_rec(-1, M, Dm, h->kpe, 4, false),
+                gemm_launch((em.pruned ? em.patch : h->patch).pick(M), M, s));
   const double ln_bytes = double(M) * Dm * (4 + 2);
   for (int l = 0; l < d.layers; ++l) {
     const VitLayerPack& lp = vm.layers[l];

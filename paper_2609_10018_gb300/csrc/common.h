@@ -110,6 +110,7 @@ struct GemmArgs {
   int cv_ho, cv_wo, cv_bw, cv_bh, cv_nb;     // output size and the pixel block of one M tile
   int cv_batch;                              // images in this launch (set at launch)
   int cv_a_bytes;                            // bytes one A tile load delivers
+  int resid_row_mod;                         // > 0: periodic residual source (gemm_set_residual_source)
 };
 
 struct GemmPlan {
@@ -152,7 +153,10 @@ struct GemmPlanSet {
 // Residual epilogues: read the addend from src [M_cap, ldo] (fp32 for
 // RESID_F32, 16-bit for the RESID_RELU ones) instead of the output
 // (out = src + acc + bias). The 16-bit residual epilogues need it.
-elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap);
+// row_period > 0: the addend repeats every row_period rows and src holds
+// M_cap >= row_period + 128 of them; output row r adds src row r mod period
+// (a tile starting at m0 reads rows m0 mod period ... + 127).
+elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap, int row_period = 0);
 // Implicit-GEMM k x k convolution (stride, padding `pad`) of the f16 NHWC
 // input x [B_cap, H, W, C] (C % 8 == 0) with W [N, k * k * Cp] f16, Cp = C
 // rounded up to 64 (zero columns), out = epi(conv + bias) f16 [B_cap, Ho, Wo,

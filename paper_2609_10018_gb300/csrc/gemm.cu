@@ -80,6 +80,14 @@ struct EpiTraits {
   static constexpr int cw = f32 ? 32 : 64;  // columns per 128-byte staging chunk
 };
 
+// Row of the residual source that a tile starting at output row m0 reads: the
+// same row, or for a periodic source (resid_row_mod rows per period, stored
+// for enough periods that any 128 consecutive rows from a start below the
+// period are present) the row m0 mod period.
+__device__ __forceinline__ int resid_row(const GemmArgs& a, int m0) {
+  return a.resid_row_mod > 0 ? m0 % a.resid_row_mod : m0;
+}
+
 template <int EPI>
 __device__ __forceinline__ float epi_act(float v) {
   if constexpr (EPI == EPI_BIAS_GELU_BF16) return gelu(v);
@@ -396,7 +404,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       if (elected) {
         for (int e = 0; e < E && pf.valid; ++e) {
           mbar_expect_tx(&rfull[e], CBUF);
-          tma_load_2d(sC + e * CBUF, &tmR, &rfull[e], (pf.t % nt) * bn + pf.c * CW, (pf.t / nt) * TM + rank * BM);
+          tma_load_2d(sC + e * CBUF, &tmR, &rfull[e], (pf.t % nt) * bn + pf.c * CW,
+                      resid_row(args, (pf.t / nt) * TM + rank * BM));
           pf.advance(tiles, nt, bn, CW, N);
           ++loads;
         }
@@ -525,7 +534,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               const int ep = e == 0 ? E - 1 : e - 1;  // buffer of the previous chunk
               mbar_expect_tx(&rfull[ep], CBUF);
               tma_load_2d(sC + ep * CBUF, &tmR, &rfull[ep], (pf.t % nt) * bn + pf.c * CW,
-                          (pf.t / nt) * TM + rank * BM);
+                          resid_row(args, (pf.t / nt) * TM + rank * BM));
               pf.advance(tiles, nt, bn, CW, N);
               ++loads;
             }
@@ -892,13 +901,18 @@ elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W
   return ELASTO_OK;
 }
 
-elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap) {
+elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap, int row_period) {
   const bool f32 = p && p->epi == EPI_BIAS_RESID_F32;
   const bool r16 = p && (p->epi == EPI_BIAS_RESID_RELU_BF16 || p->epi == EPI_BIAS_RESID_RELU_F16);
   if (!p || !p->valid || !(f32 || r16) || !src) {
     set_error("gemm_set_residual_source: needs a residual plan and a source");
     return ELASTO_ERR_INVALID_ARG;
   }
+  if (row_period < 0 || (row_period > 0 && (p->args.conv || M_cap < row_period + BM))) {
+    set_error("gemm_set_residual_source: a periodic source needs period + 128 rows and a plain GEMM");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  p->args.resid_row_mod = row_period;
   const int ldo = p->args.ldo;
   if (!encode_tmap_2d(&p->tmR, src, ldo, M_cap, static_cast<uint64_t>(ldo) * (f32 ? 4 : 2), f32 ? 32 : 64, BM,
                       f32)) {

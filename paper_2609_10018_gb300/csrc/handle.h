@@ -39,7 +39,8 @@ struct VitEmbed {
   float *patch_b = nullptr, *cls = nullptr, *pos = nullptr;  // [d_pad], [d_pad], [n, d_pad]
   std::vector<float*> ln1_w, ln1_b, ln2_w, ln2_b, proj_b, fc2_b;  // per layer, [d_pad]
   float *norm_w = nullptr, *norm_b = nullptr, *head_w = nullptr;  // [d_pad], [d_pad], [C, d_pad]
-  GemmPlanSet patch;  // pruned modes: patch rows -> X past the class token, + position embedding
+  float* addend = nullptr;  // per-token addend of the patch projection, [k * n, d_pad] (see elasto_s::tok_addend)
+  GemmPlanSet patch;        // pruned modes: the patch projection at width d_pad
 };
 
 struct VitMode {
@@ -67,7 +68,11 @@ struct elasto_s {
   // workspace
   float* X = nullptr;
   elasto::bf16 *Y = nullptr, *QKV = nullptr, *O = nullptr, *H = nullptr, *P = nullptr;
-  float* tok_addend = nullptr;  // [max_batch * n, d] addend of the patch projection
+  // Per-token addend of the patch projection (cls + pos[0] on class tokens,
+  // pos[t] + b_pe on patch tokens) for k = 1 + ceil(128 / n) images: it is
+  // the same for every image, and the patch GEMM reads row r mod n of it.
+  float* tok_addend = nullptr;  // [k * n, d]
+  int addend_rows = 0;          // k * n
   void* img_stage = nullptr;
   float* logit_stage = nullptr;
   int* status = nullptr;
