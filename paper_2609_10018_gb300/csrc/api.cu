@@ -367,7 +367,10 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       VitLayerPack& lp = h->modes[m].layers[l];
       lp.w = 64 * modes[m].n_heads_kept[l];
       lp.f = modes[m].n_mlp_kept[l];
-      lp.f_pad = (lp.f + 7) / 8 * 8;
+      // per-mode packs pad the MLP width to 64 channels: the rows of H and W2
+      // (and the GELU epilogue's tiles) then start on 128-byte boundaries;
+      // a prefix of the shared copy keeps f (a multiple of 8)
+      lp.f_pad = shared ? lp.f : (lp.f + 63) / 64 * 64;
       lp.ld_proj = shared ? 64 * static_cast<int>(h->perm_h[l].size()) : lp.w;
       lp.ld_fc2 = shared ? static_cast<int>(h->perm_f[l].size()) : lp.f_pad;
       wmax = std::max(wmax, lp.w);

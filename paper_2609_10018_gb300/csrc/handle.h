@@ -12,7 +12,7 @@ namespace elasto {
 struct VitLayerPack {
   int w = 0;       // kept heads * 64
   int f = 0;       // kept MLP channels
-  int f_pad = 0;   // f rounded up to a multiple of 8 (zero rows/cols; GELU(0) = 0)
+  int f_pad = 0;   // f, or f rounded up to 64 in a per-mode pack (zero rows/cols; GELU(0) = 0)
   int ld_proj = 0; // row stride of proj_w (w, or 64 x heads of the shared copy)
   int ld_fc2 = 0;  // row stride of fc2_w (f_pad, or the shared copy's channels)
   bf16* qkv_w = nullptr;
