@@ -155,34 +155,69 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
 // writes group t % 19 of output pixel t / 19 as one 16-byte store, so a warp
 // writes 512 contiguous bytes; the 8 source values of a group are at most
 // two image rows apart and mostly adjacent.
+// Stem gather: one CTA per output row (image b, row oy). The seven input rows
+// the row's 7x7/2 windows cover are staged once in shared memory as f16
+// (zero outside the image, three zero columns each side), then the CTA writes
+// the Wo gathered rows [Wo, 152] ((ky, kx, c) columns, 147 padded to 152) with
+// coalesced 16-byte stores.
+constexpr int kStemWmax = 1024;  // 7 x (W + 6) x 3 f16 of shared memory: <= 43 KB
+constexpr int kStemThreads = 13 * (kStemKp / 8);  // 247: a whole number of 19-group pixels
 template <typename T>
-__global__ void __launch_bounds__(256) stem_im2col_kernel(const T* __restrict__ src, int H, int W, int Ho, int Wo,
-                                                          size_t rows, uint4* __restrict__ dst) {
+__global__ void __launch_bounds__(kStemThreads) stem_im2col_kernel(const T* __restrict__ src, int H, int W, int Ho, int Wo,
+                                                          uint4* __restrict__ dst) {
   pdl_wait();
   pdl_trigger();
   constexpr int G = kStemKp / 8;
-  const size_t total = rows * G;
-  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
-       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
-    const size_t row = t / G;
-    const int g = static_cast<int>(t - row * G);
-    const int ox = static_cast<int>(row % Wo);
-    const size_t r2 = row / Wo;
-    const int oy = static_cast<int>(r2 % Ho);
-    const size_t b = r2 / Ho;
-    const T* img = src + b * H * W * 3;
-    float v[8];
+  extern __shared__ uint16_t tile_raw[];  // [ky][(ix + 3) * 3 + c], f16 bits
+  const int oy = static_cast<int>(blockIdx.x % Ho);
+  const size_t b = blockIdx.x / Ho;
+  const int wp = (W + 6) * 3;
+  // eight independent loads per thread in flight before their stores
+  constexpr int U = 8;
+  for (int i0 = threadIdx.x; i0 < 7 * wp; i0 += U * blockDim.x) {
+    float v[U];
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int k = g * 8 + i;
-      const int tap = k / 3, c = k - 3 * tap;
-      const int ky = tap / 7, kx = tap - 7 * ky;
-      const int iy = 2 * oy - 3 + ky, ix = 2 * ox - 3 + kx;
-      v[i] = (k < kStemK && iy >= 0 && iy < H && ix >= 0 && ix < W)
-                 ? static_cast<float>(img[(static_cast<size_t>(iy) * W + ix) * 3 + c])
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      const int ky = i / wp, j = i - ky * wp;
+      const int iy = 2 * oy - 3 + ky, ix = j / 3 - 3;
+      v[u] = (i < 7 * wp && iy >= 0 && iy < H && ix >= 0 && ix < W)
+                 ? static_cast<float>(src[(b * H + iy) * W * 3 + (j - 9)])
                  : 0.0f;
     }
-    dst[t] = make_uint4(pack2(v[0], v[1]), pack2(v[2], v[3]), pack2(v[4], v[5]), pack2(v[6], v[7]));
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const int i = i0 + u * blockDim.x;
+      if (i < 7 * wp) {
+        const __half hv = __float2half_rn(v[u]);
+        tile_raw[i] = *reinterpret_cast<const uint16_t*>(&hv);
+      }
+    }
+  }
+  __syncthreads();
+  // The CTA has 13 x 19 threads: thread T always builds column group
+  // g = T % 19 (columns 8g .. 8g + 7) of pixels ox = T / 19 + 13 i, so its
+  // eight shared-memory offsets are computed once; consecutive threads still
+  // write consecutive 16-byte pieces of the output rows.
+  const int g = threadIdx.x % G, ox0 = threadIdx.x / G;
+  int off[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) {
+    const int k = g * 8 + e;
+    const int tap = k / 3, c = k - 3 * tap, ky = tap / 7, kx = tap - 7 * ky;
+    off[e] = k < kStemK ? ky * wp + kx * 3 + c : -1;
+  }
+  uint4* out = dst + (b * Ho + oy) * static_cast<size_t>(Wo) * G;
+  for (int ox = ox0; ox < Wo; ox += kStemThreads / G) {
+    const uint16_t* base = tile_raw + 6 * ox;
+    uint32_t u[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const uint32_t lo = off[2 * q] >= 0 ? base[off[2 * q]] : 0u;
+      const uint32_t hi = off[2 * q + 1] >= 0 ? base[off[2 * q + 1]] : 0u;
+      u[q] = lo | (hi << 16);
+    }
+    out[ox * G + g] = make_uint4(u[0], u[1], u[2], u[3]);
   }
 }
 
@@ -249,11 +284,12 @@ __device__ __forceinline__ float warp_sum32(float v) {
   return v;
 }
 
-constexpr int FC_IMGS = 8, FC_CLASSES = 16;
+constexpr int FC_IMGS = 8, FC_CPW = 4, FC_CLASSES = 8 * FC_CPW;
 
 // logits[b, c] = pooled[b, :] . Wf[c, :] + bf[c] in fp32. grid (ceil(B / 8),
-// ceil(C / 16)), 256 threads: each warp takes two classes for 8 images; the
-// classifier row is read 4 float4 at a time so several requests are in flight.
+// ceil(C / 32)), 256 threads: each warp computes 4 classes x 8 images at once,
+// so every pooled float4 it loads feeds 16 FMAs and every classifier float4
+// 32 (the pooled rows are read from L1 once per 4 classes, not per class).
 __global__ void __launch_bounds__(256) fc_kernel(const float* __restrict__ pooled, int B, int d,
                                                  const float* __restrict__ Wf, const float* __restrict__ bf, int C,
                                                  float* __restrict__ logits) {
@@ -262,31 +298,38 @@ __global__ void __launch_bounds__(256) fc_kernel(const float* __restrict__ poole
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b0 = blockIdx.x * FC_IMGS;
   const int nimg = min(FC_IMGS, B - b0);
-  const int c0 = blockIdx.y * FC_CLASSES;
-  for (int cc = warp; cc < FC_CLASSES; cc += 8) {
-    const int cls = c0 + cc;
-    if (cls >= C) break;
-    const float* wr = Wf + static_cast<size_t>(cls) * d;
-    float acc[FC_IMGS];
+  const int c0 = blockIdx.y * FC_CLASSES + warp * FC_CPW;
+  if (c0 >= C) return;
+  const float* wr[FC_CPW];
 #pragma unroll
-    for (int i = 0; i < FC_IMGS; ++i) acc[i] = 0.0f;
-#pragma unroll 4
-    for (int c = lane * 4; c < d; c += 128) {
-      const float4 wv = *reinterpret_cast<const float4*>(wr + c);
+  for (int j = 0; j < FC_CPW; ++j) wr[j] = Wf + static_cast<size_t>(min(c0 + j, C - 1)) * d;
+  float acc[FC_CPW][FC_IMGS];
 #pragma unroll
-      for (int i = 0; i < FC_IMGS; ++i) {
-        if (i < nimg) {
-          const float4 yv = *reinterpret_cast<const float4*>(pooled + static_cast<size_t>(b0 + i) * d + c);
-          acc[i] += wv.x * yv.x + wv.y * yv.y + wv.z * yv.z + wv.w * yv.w;
-        }
-      }
-    }
+  for (int j = 0; j < FC_CPW; ++j)
+#pragma unroll
+    for (int i = 0; i < FC_IMGS; ++i) acc[j][i] = 0.0f;
+#pragma unroll 2
+  for (int c = lane * 4; c < d; c += 128) {
+    float4 wv[FC_CPW];
+#pragma unroll
+    for (int j = 0; j < FC_CPW; ++j) wv[j] = *reinterpret_cast<const float4*>(wr[j] + c);
 #pragma unroll
     for (int i = 0; i < FC_IMGS; ++i) {
-      const float v = warp_sum32(acc[i]);
-      if (lane == 0 && i < nimg) logits[static_cast<size_t>(b0 + i) * C + cls] = v + bf[cls];
+      if (i < nimg) {
+        const float4 yv = *reinterpret_cast<const float4*>(pooled + static_cast<size_t>(b0 + i) * d + c);
+#pragma unroll
+        for (int j = 0; j < FC_CPW; ++j)
+          acc[j][i] += wv[j].x * yv.x + wv[j].y * yv.y + wv[j].z * yv.z + wv[j].w * yv.w;
+      }
     }
   }
+#pragma unroll
+  for (int j = 0; j < FC_CPW; ++j)
+#pragma unroll
+    for (int i = 0; i < FC_IMGS; ++i) {
+      const float v = warp_sum32(acc[j][i]);
+      if (lane == 0 && i < nimg && c0 + j < C) logits[static_cast<size_t>(b0 + i) * C + c0 + j] = v + bf[c0 + j];
+    }
 }
 
 unsigned grid_for(size_t n) {
@@ -296,15 +339,16 @@ unsigned grid_for(size_t n) {
 
 cudaError_t stem_im2col_launch(const void* images, int dtype, int B, int H, int W, int Ho, int Wo, __half* dst,
                                cudaStream_t s) {
-  const size_t rows = static_cast<size_t>(B) * Ho * Wo;
-  if (rows == 0) return cudaSuccess;
-  const unsigned blocks = grid_for(rows * (kStemKp / 8));
+  if (B <= 0 || Ho <= 0 || Wo <= 0) return cudaSuccess;
+  if (W > kStemWmax) return cudaErrorInvalidValue;
+  const unsigned blocks = static_cast<unsigned>(B) * Ho;
+  const size_t smem = size_t(7) * (W + 6) * 3 * 2;
   uint4* d = reinterpret_cast<uint4*>(dst);
   if (dtype == ELASTO_BF16)
-    return launch_pdl(stem_im2col_kernel<bf16>, dim3(blocks), dim3(256), 0, s, static_cast<const bf16*>(images), H, W,
-                      Ho, Wo, rows, d);
-  return launch_pdl(stem_im2col_kernel<float>, dim3(blocks), dim3(256), 0, s, static_cast<const float*>(images), H,
-                    W, Ho, Wo, rows, d);
+    return launch_pdl(stem_im2col_kernel<bf16>, dim3(blocks), dim3(kStemThreads), smem, s,
+                      static_cast<const bf16*>(images), H, W, Ho, Wo, d);
+  return launch_pdl(stem_im2col_kernel<float>, dim3(blocks), dim3(kStemThreads), smem, s,
+                    static_cast<const float*>(images), H, W, Ho, Wo, d);
 }
 
 // ---------------------------------------------------------------- host packing
@@ -371,8 +415,8 @@ elasto_launch_record gemm_record(int layer, int M, int N, int K, bool resid) {
 
 elasto_status cnn_check_inputs(const elasto_model_desc* d, const elasto_weights* w, const elasto_mode_tables* modes,
                                int n_modes) {
-  if (d->img_c != 3 || d->img_h < 32 || d->img_w < 32 || d->classes < 1 || d->img_h > 4096 || d->img_w > 4096) {
-    set_error("elasto_create: ResNet-50 needs img_c = 3, 32 <= img_h, img_w <= 4096 and classes >= 1");
+  if (d->img_c != 3 || d->img_h < 32 || d->img_w < 32 || d->classes < 1 || d->img_h > 4096 || d->img_w > 1024) {
+    set_error("elasto_create: ResNet-50 needs img_c = 3, 32 <= img_h <= 4096, 32 <= img_w <= 1024, classes >= 1");
     return ELASTO_ERR_INVALID_ARG;
   }
   if (w->n_tensors != n_tensors_expected()) {

@@ -343,13 +343,14 @@ cudaError_t token_addend_launch(const float* cls, const float* pos, const float*
 // ---------------------------------------------------------------- classifier
 namespace {
 
-constexpr int HEAD_IMGS = 8;      // class-token rows per CTA
-constexpr int HEAD_CLASSES = 16;  // classes per CTA (two per warp)
+constexpr int HEAD_IMGS = 8;                  // class-token rows per CTA
+constexpr int HEAD_CPW = 4;                   // classes per warp, computed together
+constexpr int HEAD_CLASSES = 8 * HEAD_CPW;    // classes per CTA
 
-// grid (ceil(B / 8), ceil(C / 16)), 256 threads: LayerNorm of up to 8 class
-// tokens into shared memory (fp32), then each warp computes 2 classes x 8
-// images of dot products. The classifier row's loads are issued 4 float4 at a
-// time, so a warp has several HBM/L2 requests in flight instead of one.
+// grid (ceil(B / 8), ceil(C / 32)), 256 threads: LayerNorm of up to 8 class
+// tokens into shared memory (fp32), then each warp computes 4 classes x 8
+// images of dot products at once: every normalised float4 it reads from shared
+// memory feeds 16 FMAs, every classifier float4 32.
 // d is the row width of X and Wh; the LayerNorm statistics cover the first
 // d_true channels (the rest are the zero padding of a pruned width).
 __global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, int B, int n, int d, int d_true,
@@ -376,31 +377,38 @@ __global__ void __launch_bounds__(256) head_kernel(const float* __restrict__ X, 
     for (int c = lane; c < d; c += 32) sy[warp * d + c] = c < d_true ? (xr[c] - mean) * rstd * g[c] + bta[c] : 0.0f;
   }
   __syncthreads();
-  const int c0 = blockIdx.y * HEAD_CLASSES;
-  for (int cc = warp; cc < HEAD_CLASSES; cc += 8) {
-    const int cls = c0 + cc;
-    if (cls >= C) break;
-    const float* wr = Wh + static_cast<size_t>(cls) * d;
-    float acc[HEAD_IMGS];
+  const int c0 = blockIdx.y * HEAD_CLASSES + warp * HEAD_CPW;
+  if (c0 >= C) return;
+  const float* wr[HEAD_CPW];
 #pragma unroll
-    for (int i = 0; i < HEAD_IMGS; ++i) acc[i] = 0.0f;
-#pragma unroll 4
-    for (int c = lane * 4; c < d; c += 128) {
-      const float4 wv = *reinterpret_cast<const float4*>(wr + c);
+  for (int j = 0; j < HEAD_CPW; ++j) wr[j] = Wh + static_cast<size_t>(min(c0 + j, C - 1)) * d;
+  float acc[HEAD_CPW][HEAD_IMGS];
 #pragma unroll
-      for (int i = 0; i < HEAD_IMGS; ++i) {
-        if (i < nimg) {
-          const float4 yv = *reinterpret_cast<const float4*>(sy + i * d + c);
-          acc[i] += wv.x * yv.x + wv.y * yv.y + wv.z * yv.z + wv.w * yv.w;
-        }
-      }
-    }
+  for (int j = 0; j < HEAD_CPW; ++j)
+#pragma unroll
+    for (int i = 0; i < HEAD_IMGS; ++i) acc[j][i] = 0.0f;
+#pragma unroll 2
+  for (int c = lane * 4; c < d; c += 128) {
+    float4 wv[HEAD_CPW];
+#pragma unroll
+    for (int j = 0; j < HEAD_CPW; ++j) wv[j] = *reinterpret_cast<const float4*>(wr[j] + c);
 #pragma unroll
     for (int i = 0; i < HEAD_IMGS; ++i) {
-      const float v = warp_sum(acc[i]);
-      if (lane == 0 && i < nimg) logits[static_cast<size_t>(b0 + i) * C + cls] = v + bh[cls];
+      if (i < nimg) {
+        const float4 yv = *reinterpret_cast<const float4*>(sy + i * d + c);
+#pragma unroll
+        for (int j = 0; j < HEAD_CPW; ++j)
+          acc[j][i] += wv[j].x * yv.x + wv[j].y * yv.y + wv[j].z * yv.z + wv[j].w * yv.w;
+      }
     }
   }
+#pragma unroll
+  for (int j = 0; j < HEAD_CPW; ++j)
+#pragma unroll
+    for (int i = 0; i < HEAD_IMGS; ++i) {
+      const float v = warp_sum(acc[j][i]);
+      if (lane == 0 && i < nimg && c0 + j < C) logits[static_cast<size_t>(b0 + i) * C + c0 + j] = v + bh[c0 + j];
+    }
 }
 
 }  // namespace
