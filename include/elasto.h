@@ -274,6 +274,17 @@ elasto_status elasto_saliency(const elasto_model_desc* desc, const elasto_weight
  * one ranking makes the modes nested (Eq. 8). Host-only. Errors: INVALID_ARG. */
 elasto_status elasto_topk(const float* scores, int n, int k, int32_t* out);
 
+/* L1-norm saliency of the d embedding channels of a ViT (Section 4.1: the
+ * compress stage also shrinks the hidden size of the LayerNorm and
+ * patch-embedding layers). Channel c owns the rows that write it (row c of the
+ * patch projection, and of W^O and W2 in every layer) and the columns that
+ * read it (column c of W_qkv and W1 in every layer, and of the classifier);
+ * scores_e[c] [dim] is the mean of those 2 + 4 * layers row/column averages of
+ * |w|. Same descriptor and tensor order as elasto_create; synchronous.
+ * elasto_topk on the scores gives nested embed_kept tables (Eq. 8).
+ * Errors: INVALID_ARG (not a ViT, null argument), CUDA, OOM. */
+elasto_status elasto_saliency_embed(const elasto_model_desc* desc, const elasto_weights* weights, float* scores_e);
+
 /* Test hook: copy one packed buffer of (mode, layer) to host_dst (bytes must
  * equal its size). ViT `which`: 0 qkv_w bf16 [3w,d], 1 qkv_b fp32 [3w],
  * 2 proj_w bf16 [d,w], 3 fc1_w bf16 [f,d], 4 fc1_b fp32 [f], 5 fc2_w bf16 [d,f]

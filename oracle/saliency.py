@@ -18,6 +18,12 @@ the granularity the descendant networks use, as for the kept tables):
     input slice (over w_out x 3 x 3); a channel of S_b owns conv2's output row
     (over w_in x 3 x 3) and conv3's input column (over 4w); its saliency is the
     mean of its two averages;
+  - an embedding channel c (the residual-stream width pruned with the
+    LayerNorm and patch-embedding hidden size) owns the rows that write it and
+    the columns that read it: row c of the patch projection (over C x P x P),
+    of W^O and of W2 in every layer; column c of W_qkv and of W1 in every
+    layer and of the classifier. Its saliency is the mean of those 2 + 4L
+    averages (LayerNorm gains are scales, not rows, and are left out);
   - a mode keeping k units keeps the k most salient (ties: lower index),
     listed ascending; one ranking for all modes makes the sets nested (Eq. 8).
 """
@@ -42,6 +48,20 @@ def vit_saliency(w: dict, cfg) -> tuple[np.ndarray, np.ndarray]:
         fc2 = np.abs(w[f"l{l}.fc2_w"]).mean(axis=0)           # [d_ff] columns
         fs[l] = 0.5 * (fc1 + fc2)
     return hs, fs
+
+
+def vit_embed_saliency(w: dict, cfg) -> np.ndarray:
+    """`w` widened to float64. Scores of the d embedding channels."""
+    d = cfg.dim
+    parts = [np.abs(w["patch_w"]).reshape(d, -1).mean(axis=1),   # patch projection rows
+             np.abs(w["head_w"]).mean(axis=0)]                     # classifier columns
+    for l in range(cfg.layers):
+        p = f"l{l}."
+        parts += [np.abs(w[p + "qkv_w"]).mean(axis=0),             # W_qkv columns (inputs)
+                  np.abs(w[p + "proj_w"]).mean(axis=1),            # W^O rows (outputs)
+                  np.abs(w[p + "fc1_w"]).mean(axis=0),             # W1 columns
+                  np.abs(w[p + "fc2_w"]).mean(axis=1)]             # W2 rows
+    return np.mean(parts, axis=0)
 
 
 def resnet_saliency(w: dict, blocks) -> tuple[list, list]:

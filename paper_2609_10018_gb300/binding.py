@@ -97,6 +97,7 @@ def lib() -> ctypes.CDLL:
         "elasto_select_dn": [ctypes.POINTER(DnProfile), c_int, ctypes.c_float, ctypes.c_double, ctypes.c_float,
                              ctypes.POINTER(c_int)],
         "elasto_saliency": [ctypes.POINTER(ModelDesc), ctypes.POINTER(Weights), c_void_p, c_void_p],
+        "elasto_saliency_embed": [ctypes.POINTER(ModelDesc), ctypes.POINTER(Weights), c_void_p],
         "elasto_topk": [c_void_p, c_int, c_int, c_void_p],
         "elasto_op_gemm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_int,
                            c_void_p],
@@ -298,6 +299,15 @@ def elasto_saliency(desc: ModelDesc, tensors: Sequence[np.ndarray], n_a: int, n_
     return a, b
 
 
+def elasto_saliency_embed(desc: ModelDesc, tensors: Sequence[np.ndarray]) -> np.ndarray:
+    """L1 saliency of the ViT's embedding channels, computed on the GPU."""
+    keep = _Keep()
+    w = weights_struct(keep, tensors)
+    e = np.zeros(desc.dim, np.float32)
+    _check(lib().elasto_saliency_embed(ctypes.byref(desc), ctypes.byref(w), e.ctypes.data), "elasto_saliency_embed")
+    return e
+
+
 def elasto_topk(scores: np.ndarray, k: int) -> np.ndarray:
     s = np.ascontiguousarray(scores, dtype=np.float32)
     out = np.zeros(k, np.int32)
@@ -305,18 +315,24 @@ def elasto_topk(scores: np.ndarray, k: int) -> np.ndarray:
     return out
 
 
-def saliency_tables_vit(cfg, weights, names=None):
+def saliency_tables_vit(cfg, weights, names=None, embed_widths=None):
     """Kept tables for cfg's modes from the GPU saliency: per layer the most
-    salient heads / MLP channels (nested across modes, Eq. 8)."""
+    salient heads / MLP channels, and with embed_widths (one per mode, None =
+    all) the most salient embedding channels; nested across modes (Eq. 8)."""
     from . import synth
     names = names or synth.vit_weight_names(cfg)
-    a, b = elasto_saliency(vit_desc(cfg, 1), [weights[k] for k in names], cfg.layers * cfg.heads,
-                           cfg.layers * cfg.mlp)
+    tensors = [weights[k] for k in names]
+    a, b = elasto_saliency(vit_desc(cfg, 1), tensors, cfg.layers * cfg.heads, cfg.layers * cfg.mlp)
     a = a.reshape(cfg.layers, cfg.heads)
     b = b.reshape(cfg.layers, cfg.mlp)
-    return [{"heads": [elasto_topk(a[l], kh) for l in range(cfg.layers)],
-             "mlp": [elasto_topk(b[l], kf) for l in range(cfg.layers)]}
-            for kh, kf in zip(cfg.mode_heads, cfg.mode_mlp)]
+    tables = [{"heads": [elasto_topk(a[l], kh) for l in range(cfg.layers)],
+               "mlp": [elasto_topk(b[l], kf) for l in range(cfg.layers)]}
+              for kh, kf in zip(cfg.mode_heads, cfg.mode_mlp)]
+    if embed_widths is not None:
+        e = elasto_saliency_embed(vit_desc(cfg, 1), tensors)
+        for t, k in zip(tables, embed_widths):
+            t["embed"] = None if k is None else elasto_topk(e, k)
+    return tables
 
 
 def elasto_op_gemm(stream, A, W, bias, out, resid, M, N, K, epilogue, status=0) -> None:

@@ -9,7 +9,9 @@
 //                      input columns of W^O (the paper's rows of W^O);
 //   ViT MLP channel c: row c of W1 and column c of W2;
 //   ResNet S_a channel: conv1's output row and conv2's input slice;
-//   ResNet S_b channel: conv2's output row and conv3's input column.
+//   ResNet S_b channel: conv2's output row and conv3's input column;
+//   ViT embedding channel: the rows that write it (patch projection, W^O, W2)
+//                      and the columns that read it (W_qkv, W1, classifier).
 // The reductions are memory-bound passes over the weights (each weight read
 // once): a warp per row for row averages, a thread per column for column
 // averages, fp32 sums of |w|.
@@ -174,6 +176,53 @@ elasto_status elasto_saliency(const elasto_model_desc* d, const elasto_weights* 
   }
   set_error("elasto_saliency: unknown arch");
   return ELASTO_ERR_INVALID_ARG;
+}
+
+elasto_status elasto_saliency_embed(const elasto_model_desc* d, const elasto_weights* w, float* scores_e) {
+  clear_error();
+  if (!d || !w || !w->tensors || !scores_e || d->arch != ELASTO_ARCH_VIT ||
+      (d->weight_dtype != ELASTO_F32 && d->weight_dtype != ELASTO_BF16)) {
+    set_error("elasto_saliency_embed: null argument, not a ViT, or bad weight_dtype");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int L = d->layers, D = d->dim, H = d->heads, F = d->mlp, C = d->classes;
+  if (L <= 0 || H <= 0 || D != 64 * H || F <= 0 || C <= 0 || d->patch <= 0 || d->img_c <= 0 ||
+      w->n_tensors != 8 + 12 * L) {
+    set_error("elasto_saliency_embed: inconsistent ViT descriptor or tensor count");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  for (int i = 0; i < w->n_tensors; ++i)
+    if (!w->tensors[i]) {
+      set_error("elasto_saliency_embed: null weight tensor " + std::to_string(i));
+      return ELASTO_ERR_INVALID_ARG;
+    }
+  // The rows that write channel c and the columns that read it: patch
+  // projection rows, classifier columns, and per layer W_qkv / W1 columns and
+  // W^O / W2 rows; the score is the mean of those 2 + 4L averages.
+  Reducer red{d->weight_dtype};
+  std::vector<double> sum(D, 0.0);
+  std::vector<float> a;
+  auto add = [&]() {
+    for (int c = 0; c < D; ++c) sum[c] += a[c];
+  };
+  const int kpe = d->patch * d->patch * d->img_c;
+  ELASTO_CUDA_TRY(red.reduce(w->tensors[0], D, kpe, true, a));  // patch_w [d, C, P, P] rows
+  add();
+  ELASTO_CUDA_TRY(red.reduce(w->tensors[4 + 12 * L + 2], C, D, false, a));  // head_w [C, d] columns
+  add();
+  for (int l = 0; l < L; ++l) {
+    const int t0 = 4 + 12 * l;
+    ELASTO_CUDA_TRY(red.reduce(w->tensors[t0 + 2], 3 * D, D, false, a));  // W_qkv columns
+    add();
+    ELASTO_CUDA_TRY(red.reduce(w->tensors[t0 + 4], D, D, true, a));      // W^O rows
+    add();
+    ELASTO_CUDA_TRY(red.reduce(w->tensors[t0 + 8], F, D, false, a));     // W1 columns
+    add();
+    ELASTO_CUDA_TRY(red.reduce(w->tensors[t0 + 10], D, F, true, a));     // W2 rows
+    add();
+  }
+  for (int c = 0; c < D; ++c) scores_e[c] = static_cast<float>(sum[c] / (2 + 4 * L));
+  return ELASTO_OK;
 }
 
 elasto_status elasto_topk(const float* scores, int n, int k, int32_t* out) {

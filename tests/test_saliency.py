@@ -9,7 +9,7 @@ import pytest
 
 from oracle import resnet as orr
 from oracle import vit as ov
-from oracle.saliency import resnet_saliency, top_k, vit_saliency
+from oracle.saliency import resnet_saliency, top_k, vit_embed_saliency, vit_saliency
 from paper_2609_10018_gb300 import binding, synth
 
 TINY_BF16 = synth.vit_small_variant(synth.TINY, dtype=synth.BF16)
@@ -30,6 +30,24 @@ def test_oracle_finds_planted_head_and_channel():
     rows = [qkv[b * d + j * 64 + r].mean() for b in range(3) for r in range(64)] + \
            [proj[:, j * 64 + r].mean() for r in range(64)]
     assert abs(hs[l, j] - np.mean(rows)) < 1e-15
+
+
+def test_oracle_embedding_saliency_planted_and_closed_form():
+    cfg = synth.TINY
+    w = ov.widen_all(synth.make_vit_weights(cfg))
+    w["l2.fc2_w"][41] *= 30.0                         # channel 41: its W2 row (an output of the block)
+    w["l4.qkv_w"][:, 99] *= 30.0                      # channel 99: its W_qkv column (an input)
+    e = vit_embed_saliency(w, cfg)
+    assert set(top_k(e, 2).tolist()) == {41, 99}
+    # closed form for one channel: mean of its 2 + 4L row / column averages
+    c, d = 7, cfg.dim
+    parts = [np.abs(w["patch_w"][c]).mean(), np.abs(w["head_w"][:, c]).mean()]
+    for l in range(cfg.layers):
+        parts += [np.abs(w[f"l{l}.qkv_w"][:, c]).mean(), np.abs(w[f"l{l}.proj_w"][c]).mean(),
+                  np.abs(w[f"l{l}.fc1_w"][:, c]).mean(), np.abs(w[f"l{l}.fc2_w"][c]).mean()]
+    assert len(parts) == 2 + 4 * cfg.layers
+    assert abs(e[c] - np.mean(parts)) < 1e-15
+    assert e.shape == (d,)
 
 
 def test_oracle_top_k_rules():
@@ -80,6 +98,38 @@ def test_gpu_vit_saliency_matches_oracle(cfg):
             if got != ref:
                 cut = np.sort(fs[l])[::-1][kf - 1: kf + 1]
                 assert abs(cut[0] - cut[1]) <= 1e-5 * abs(cut[0])
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("cfg", [synth.TINY, synth.VIT_S], ids=lambda c: c.name)
+def test_gpu_embedding_saliency_matches_oracle(cfg):
+    w = synth.make_vit_weights(cfg)
+    e = binding.elasto_saliency_embed(binding.vit_desc(cfg, 1), [w[k] for k in synth.vit_weight_names(cfg)])
+    ref = vit_embed_saliency(ov.widen_all(w), cfg)
+    assert np.allclose(e, ref, rtol=2e-5, atol=0)
+
+
+@pytest.mark.gpu
+def test_gpu_model_from_embedding_saliency_tables():
+    """Heads, MLP channels and embedding channels all chosen by the GPU
+    saliency; every mode matches the oracle."""
+    from helpers import dev, empty_dev, rel_err, stream_handle
+    import torch
+    cfg = synth.TINY
+    w = synth.make_vit_weights(cfg)
+    tables = binding.saliency_tables_vit(cfg, w, embed_widths=[None, 120])
+    assert len(tables[1]["embed"]) == 120
+    wide = ov.widen_all(w)
+    img = synth.make_images(cfg, 16)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=16) as model:
+        x = dev(img)
+        out = empty_dev((16, cfg.classes), torch.float32)
+        for m, t in enumerate(tables):
+            model.set_mode(m)
+            model.forward(stream_handle(), x.data_ptr(), 16, out.data_ptr())
+            model.sync_status(stream_handle())
+            ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img, embed_kept=t.get("embed"))
+            assert rel_err(out.cpu().numpy().astype(np.float64), ref) <= 1e-2
 
 
 @pytest.mark.gpu
