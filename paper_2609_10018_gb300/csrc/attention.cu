@@ -9,7 +9,9 @@
 // heads concatenated in the same order (the K axis of the packed W^O).
 //
 // Persistent kernel; a work item is one (image, kept head) and needs at most
-// two 128-query tiles (n <= 256). Roles:
+// two 128-query tiles (n <= 256). Items run from the last image to the first:
+// the QKV GEMM wrote its rows in increasing order, so the most recent (still
+// in L2) are read first. Roles:
 //   warp 0      TMA producer: Q tiles, K and V of the next item into one of
 //               two shared-memory slots (3-D maps: rows past n read as zero),
 //               so loads of item i+1 overlap the math of item i;
@@ -94,7 +96,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       int i = 0;
       for (int item = blockIdx.x; item < items; item += gridDim.x, ++i) {
-        const int slot = i & 1, b = item / heads, jj = item - b * heads;
+        const int slot = i & 1, b = (items - 1 - item) / heads, jj = (items - 1 - item) - b * heads;
         if (!mbar_wait(&slot_empty[slot], ((i >> 1) & 1) ^ 1)) {
           ok = false;
           break;
@@ -174,7 +176,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       int i = 0;
       for (int item = blockIdx.x; item < items; item += gridDim.x, ++i) {
         const uint32_t ph = i & 1;
-        const int b = item / heads, jj = item - b * heads;
+        const int b = (items - 1 - item) / heads, jj = (items - 1 - item) - b * heads;
         if (!mbar_wait(&s_full[t], ph)) {
           if (lane == 0) record_status(status, ELASTO_ERR_TIMEOUT);
           break;
