@@ -73,6 +73,16 @@ elasto_status elasto_op_conv2d(void* stream, const void* x, int B, int H, int W,
 elasto_status elasto_op_attention(void* stream, const void* qkv, void* out, int batch, int n, int heads,
                                   int* status_device);
 
+/* Self-test of the bounded device-side wait that every kernel above (and the
+ * forward's kernels) uses instead of an unbounded spin: one thread waits on an
+ * mbarrier of one arrival. armed != 0: the arrival is made first and the wait
+ * returns at once (status untouched). armed == 0: nothing arrives, the wait
+ * gives up after its limit (1 s), the kernel writes ELASTO_ERR_TIMEOUT to
+ * *status_device (if it still holds 0) and returns; the context stays usable.
+ * *elapsed_ns_device (uint64) receives the time waited. */
+elasto_status elasto_op_bounded_wait(void* stream, int armed, int* status_device,
+                                     unsigned long long* elapsed_ns_device);
+
 #ifdef __cplusplus
 }
 #endif

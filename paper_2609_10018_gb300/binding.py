@@ -106,6 +106,7 @@ def lib() -> ctypes.CDLL:
         "elasto_op_layernorm": [c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int],
         "elasto_op_softmax": [c_void_p, c_void_p, c_void_p, c_int, c_int],
         "elasto_op_attention": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p],
+        "elasto_op_bounded_wait": [c_void_p, c_int, c_void_p, c_void_p],
     }
     for name, args in sig.items():
         f = getattr(L, name)
@@ -354,6 +355,10 @@ def elasto_op_softmax(stream, x, y, rows, cols) -> None:
 
 def elasto_op_attention(stream, qkv, out, batch, n, heads, status=0) -> None:
     _check(lib().elasto_op_attention(stream, qkv, out, batch, n, heads, status), "elasto_op_attention")
+
+
+def elasto_op_bounded_wait(stream, armed: bool, status, elapsed_ns) -> None:
+    _check(lib().elasto_op_bounded_wait(stream, 1 if armed else 0, status, elapsed_ns), "elasto_op_bounded_wait")
 
 
 # ----------------------------------------------------------------------------

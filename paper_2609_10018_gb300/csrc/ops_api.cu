@@ -3,10 +3,47 @@
 // step at arbitrary (odd, ragged) shapes.
 #include "common.h"
 #include "elasto_internal.h"
+#include "ptx.cuh"
 
 using namespace elasto;
 
+namespace {
+
+// The bounded wait every kernel uses (mbar_wait: a time limit, then false),
+// on an mbarrier of one arrival. armed != 0: that arrival is made first, so
+// the wait returns at once; armed == 0: nothing ever arrives, the wait gives
+// up after its limit and the kernel records ELASTO_ERR_TIMEOUT in *status
+// and returns, leaving the context usable. *elapsed_ns: how long it waited.
+__global__ void bounded_wait_kernel(int armed, int* status, unsigned long long* elapsed_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x != 0) return;
+  mbar_init(&bar, 1);
+  fence_barrier_init();
+  if (armed) mbar_arrive(&bar);
+  const uint64_t t0 = global_timer_ns();
+  const bool ok = mbar_wait(&bar, 0);
+  *elapsed_ns = global_timer_ns() - t0;
+  if (!ok) record_status(status, ELASTO_ERR_TIMEOUT);
+}
+
+}  // namespace
+
 extern "C" {
+
+elasto_status elasto_op_bounded_wait(void* stream, int armed, int* status_device,
+                                     unsigned long long* elapsed_ns_device) {
+  clear_error();
+  if (!status_device || !elapsed_ns_device) {
+    set_error("elasto_op_bounded_wait: null argument");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  elasto_status st = check_device();
+  if (st != ELASTO_OK) return st;
+  bounded_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(armed, status_device, elapsed_ns_device);
+  ELASTO_CUDA_TRY(cudaGetLastError());
+  return ELASTO_OK;
+}
+
 
 elasto_status elasto_op_gemm(void* stream, const void* A, const void* W, const float* bias, void* out,
                              const void* resid, int M, int N, int K, int epilogue, int* status_device) {

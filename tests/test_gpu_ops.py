@@ -226,3 +226,25 @@ def test_conv2d_implicit_gemm_matches_fp64(B, H, W, C, N, k, stride, pad, relu):
     assert np.all(np.isfinite(got))
     scale = float(np.max(np.abs(ref)))
     assert np.all(np.abs(got - ref) <= 2.0 ** -10 * np.abs(ref) + 1e-4 * scale), float(np.max(np.abs(got - ref)))
+
+
+def test_bounded_wait_gives_up_and_leaves_the_context_usable():
+    """A device-side wait that nothing satisfies ends after its limit with
+    ELASTO_ERR_TIMEOUT in the status word (no trap, no hang); the next launch
+    on the same context works. An armed wait returns at once."""
+    import time
+    import torch
+    st = _status()
+    el = torch.zeros(1, dtype=torch.int64, device="cuda")
+    binding.elasto_op_bounded_wait(stream_handle(), True, st.data_ptr(), el.data_ptr())
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert int(el.item()) < 10_000_000                     # well under 10 ms
+    t0 = time.perf_counter()
+    binding.elasto_op_bounded_wait(stream_handle(), False, st.data_ptr(), el.data_ptr())
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    assert int(st.item()) == binding.ERR_TIMEOUT
+    assert 0.9e9 <= int(el.item()) <= 3e9 and wall < 10.0
+    # the context is still usable: an attention launch right after matches the oracle
+    test_attention_matches_fp64(2, 65, 2)
