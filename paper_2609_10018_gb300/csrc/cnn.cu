@@ -169,8 +169,11 @@ __global__ void __launch_bounds__(kStemThreads) stem_im2col_kernel(const T* __re
   pdl_trigger();
   constexpr int G = kStemKp / 8;
   extern __shared__ uint16_t tile_raw[];  // [ky][(ix + 3) * 3 + c], f16 bits
-  const int oy = static_cast<int>(blockIdx.x % Ho);
-  const size_t b = blockIdx.x / Ho;
+  // output rows last to first: the stem GEMM reads them first to last, so the
+  // most recently written (still in L2) are the first it reads
+  const unsigned bid = gridDim.x - 1 - blockIdx.x;
+  const int oy = static_cast<int>(bid % Ho);
+  const size_t b = bid / Ho;
   const int wp = (W + 6) * 3;
   // eight independent loads per thread in flight before their stores
   constexpr int U = 8;
@@ -230,8 +233,10 @@ __global__ void maxpool_kernel(const uint4* __restrict__ src, int H, int W, int 
   pdl_trigger();
   for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
        t += static_cast<size_t>(gridDim.x) * blockDim.x) {
-    const int c8 = static_cast<int>(t % C8);
-    const size_t p = t / C8;
+    // pixels last to first: the stem GEMM wrote its rows first to last
+    const size_t u = total - 1 - t;
+    const int c8 = static_cast<int>(u % C8);
+    const size_t p = u / C8;
     const int ox = static_cast<int>(p % Wo);
     const size_t r2 = p / Wo;
     const int oy = static_cast<int>(r2 % Ho);
@@ -251,7 +256,7 @@ __global__ void maxpool_kernel(const uint4* __restrict__ src, int H, int W, int 
         for (int j = 0; j < 8; ++j) m[j] = fmaxf(m[j], f[j]);
       }
     }
-    dst[t] = make_uint4(pack2(m[0], m[1]), pack2(m[2], m[3]), pack2(m[4], m[5]), pack2(m[6], m[7]));
+    dst[u] = make_uint4(pack2(m[0], m[1]), pack2(m[2], m[3]), pack2(m[4], m[5]), pack2(m[6], m[7]));
   }
 }
 
@@ -724,6 +729,9 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
       st = gemm_plan(&bp.conv1, xin, mi_cap, bp.w1, bp.a_pad, b.cin, bp.b1, m->t1, bp.a_pad, EPI_BIAS_RELU_F16,
                         m->status);
       if (st != ELASTO_OK) return st;
+      // conv1 reads the previous block's output, written first row to last:
+      // reading it last row first finds the most recent rows still in L2
+      bp.conv1.args.m_reverse = 1;
       st = gemm_plan_conv(&bp.conv2, m->t1, Bm, b.hin, b.win, bp.a_pad, 3, b.stride, 1, bp.w2, bp.b_pad, bp.b2, m->t2,
                           bp.b_pad, EPI_BIAS_RELU_F16, m->status);
       if (st != ELASTO_OK) return st;

@@ -111,6 +111,7 @@ struct GemmArgs {
   int cv_batch;                              // images in this launch (set at launch)
   int cv_a_bytes;                            // bytes one A tile load delivers
   int resid_row_mod;                         // > 0: periodic residual source (gemm_set_residual_source)
+  int m_reverse;                             // 1: tile rows scheduled last to first (L2 reuse of A)
 };
 
 struct GemmPlan {

@@ -80,6 +80,11 @@ struct EpiTraits {
   static constexpr int cw = f32 ? 32 : 64;  // columns per 128-byte staging chunk
 };
 
+// M-tile of the q-th tile row in the schedule: q, or mt - 1 - q when the plan
+// runs its rows last to first (m_reverse: the GEMM then reads first the rows
+// of its A operand that the previous kernel wrote last, still in L2).
+__device__ __forceinline__ int m_tile(const GemmArgs& a, int q, int mt) { return a.m_reverse ? mt - 1 - q : q; }
+
 // Row of the residual source that a tile starting at output row m0 reads: the
 // same row, or for a periodic source (resid_row_mod rows per period, stored
 // for enough periods that any 128 consecutive rows from a start below the
@@ -260,9 +265,9 @@ __global__ void __launch_bounds__(THREADS, 1)
       const uint32_t bytes =
           PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2) : (args.conv ? args.cv_a_bytes : A_STAGE) + NB * bn * BK * 2;
       for (int t = t_start; t < tiles && ok; t += t_stride) {
-        const int m0 = (t / nt) * TM + rank * BM, n0 = (t % nt) * bn;
+        const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
         int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
-        if (args.conv) conv_tile(args, t / nt, cb0, cy0, cx0);
+        if (args.conv) conv_tile(args, m_tile(args, t / nt, mt), cb0, cy0, cx0);
         for (int kb = 0; kb < nk; ++kb) {
           if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
             ok = false;
@@ -405,7 +410,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int e = 0; e < E && pf.valid; ++e) {
           mbar_expect_tx(&rfull[e], CBUF);
           tma_load_2d(sC + e * CBUF, &tmR, &rfull[e], (pf.t % nt) * bn + pf.c * CW,
-                      resid_row(args, (pf.t / nt) * TM + rank * BM));
+                      resid_row(args, m_tile(args, pf.t / nt, mt) * TM + rank * BM));
           pf.advance(tiles, nt, bn, CW, N);
           ++loads;
         }
@@ -426,7 +431,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       tc_fence_after();
-      const int m0 = (t / nt) * TM + rank * BM, n0 = (t % nt) * bn;
+      const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
       const uint32_t acc_tm = row_tm + acc * MAX_BN;
       int nvalid = 0;
       while (nvalid < cpt && n0 + nvalid * CW < N) ++nvalid;
@@ -523,7 +528,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (elected) {
           if (args.conv) {
             int cb0, cy0, cx0;
-            conv_tile(args, t / nt, cb0, cy0, cx0);
+            conv_tile(args, m_tile(args, t / nt, mt), cb0, cy0, cx0);
             tma_store_4d(&tmC, buf, n0 + c * CW, cx0, cy0, cb0);
           } else {
             tma_store_2d(&tmC, buf, n0 + c * CW, m0);
@@ -534,7 +539,7 @@ __global__ void __launch_bounds__(THREADS, 1)
               const int ep = e == 0 ? E - 1 : e - 1;  // buffer of the previous chunk
               mbar_expect_tx(&rfull[ep], CBUF);
               tma_load_2d(sC + ep * CBUF, &tmR, &rfull[ep], (pf.t % nt) * bn + pf.c * CW,
-                          resid_row(args, (pf.t / nt) * TM + rank * BM));
+                          resid_row(args, m_tile(args, pf.t / nt, mt) * TM + rank * BM));
               pf.advance(tiles, nt, bn, CW, N);
               ++loads;
             }
@@ -577,7 +582,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       tc_fence_after();
-      const int m0 = (t / nt) * TM + rank * BM, n0 = (t % nt) * bn;
+      const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
       const int row0 = m0 + q * 32;
       for (int c = 0; c < bn; c += 32) {
         if (n0 + c >= N) break;
