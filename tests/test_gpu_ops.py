@@ -171,6 +171,35 @@ def test_attention_matches_fp64(B, n, h):
     assert np.max(np.abs(got - ref)) <= 1e-2 * np.max(np.abs(ref)), float(np.max(np.abs(got - ref)))
 
 
+def test_attention_reference_raised_by_a_late_large_score():
+    """Rows whose largest score lies far beyond the first 32 keys (and far
+    above their scores): the one-pass softmax must raise its reference and
+    rescale the P it already wrote. Rows 0-5 and 130-135 attend almost
+    entirely to key 150 (q . k = 768 there, |q . k| ~ 20 elsewhere)."""
+    import torch
+    B, n, h = 2, 197, 3
+    rng = np.random.default_rng(77)
+    qkv = (rng.standard_normal((B, n, 3, h, 64)) * 0.3).astype(np.float32)
+    rows = np.r_[0:6, 130:136]
+    qkv[:, rows, 0, :, :] = 3.5
+    qkv[:, 150, 1, :, :] = 3.5
+    qkv = synth.f32_to_bf16_bits(qkv)
+    out = empty_dev((B, n, h * 64), torch.uint16)
+    st = _status()
+    dq = dev(qkv)
+    binding.elasto_op_attention(stream_handle(), dq.data_ptr(), out.data_ptr(), B, n, h, st.data_ptr())
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    q = bf16_to_f64(qkv)
+    ref = np.concatenate([ov.attention(q[:, :, 0, j], q[:, :, 1, j], q[:, :, 2, j], 64) for j in range(h)], axis=-1)
+    got = bf16_to_f64(out)
+    assert np.all(np.isfinite(got))
+    assert np.max(np.abs(got - ref)) <= 1e-2 * np.max(np.abs(ref)), float(np.max(np.abs(got - ref)))
+    # those rows are (almost) the value row of key 150
+    assert np.allclose(got[:, rows], np.concatenate([q[:, 150:151, 2, j] for j in range(h)], axis=-1)
+                       .repeat(len(rows), axis=1), atol=2e-2)
+
+
 def test_attention_full_size_sampled():
     """ViT-B shape at batch 256: 256 x 12 heads x 197 tokens; sampled images."""
     import torch
