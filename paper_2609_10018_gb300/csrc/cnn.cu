@@ -151,11 +151,8 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
 }
 
 // The stem's gather (7x7, stride 2, padding 3, 3 channels; 147 columns in
-// (ky, kx, c) order padded with zeros to 152 = 19 groups of 8). Thread t
-// writes group t % 19 of output pixel t / 19 as one 16-byte store, so a warp
-// writes 512 contiguous bytes; the 8 source values of a group are at most
-// two image rows apart and mostly adjacent.
-// Stem gather: one CTA per output row (image b, row oy). The seven input rows
+// (ky, kx, c) order padded with zeros to 152 = 19 groups of 8).
+// One CTA per output row (image b, row oy). The seven input rows
 // the row's 7x7/2 windows cover are staged once in shared memory as f16
 // (zero outside the image, three zero columns each side), then the CTA writes
 // the Wo gathered rows [Wo, 152] ((ky, kx, c) columns, 147 padded to 152) with
