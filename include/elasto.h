@@ -214,7 +214,9 @@ elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value);
  * memory-bound kernels). Events add a few microseconds per forward. */
 enum {
   ELASTO_K_PATCHIFY = 0, ELASTO_K_GEMM = 1, ELASTO_K_LAYERNORM = 2, ELASTO_K_ATTENTION = 3,
-  ELASTO_K_HEAD = 4, ELASTO_K_IM2COL = 5, ELASTO_K_POOL = 6
+  ELASTO_K_HEAD = 4,
+  ELASTO_K_IM2COL = 5, /* the CNN stem's input rearrangement (space-to-depth) */
+  ELASTO_K_POOL = 6
 };
 typedef struct {
   int kind;     /* ELASTO_K_* */

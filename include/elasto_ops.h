@@ -57,9 +57,10 @@ elasto_status elasto_op_softmax(void* stream, const float* x, float* y, int rows
  * GEMM: out f16 [B, Ho, Wo, N] = act(conv(x) + bias), Ho = (H + 2 pad - k) /
  * stride + 1 (likewise Wo), act = ReLU if relu != 0 else identity.
  *   x f16 [B, H, W, C] NHWC, C % 8 == 0;
- *   w f16 [N, k, k, Cp] with Cp = C rounded up to 64, channels >= C zero
- *     (the packed layout the ResNet path uses: one 64-channel group per
- *     k-block of the tensor-core GEMM);
+ *   w f16 [N, k, k, Cp] with Cp = 16 if C <= 16, else C rounded up to 64;
+ *     channels >= C zero (the packed layout the ResNet path uses: one
+ *     64-channel group per k-block of the tensor-core GEMM, or for at most 16
+ *     channels one tap per 16-wide k-block in the 32-byte swizzle);
  *   bias fp32 [N] or NULL. N % 2 == 0, stride 1 or 2.
  * No im2col buffer: each k-block is one 4-D TMA tile of x (padding read as
  * zeros, the stride by TMA traversal strides). */

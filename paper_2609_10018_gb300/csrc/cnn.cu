@@ -43,8 +43,13 @@ namespace {
 
 constexpr double kBnEps = 1e-5;
 constexpr int kStemC = 64;
-constexpr int kStemK = 7 * 7 * 3;  // (ky, kx, c) columns of a stem patch row
-constexpr int kStemKp = 152;       // padded to a multiple of 8
+constexpr int kStemK = 7 * 7 * 3;  // multiply-adds per output value of the 7x7 stem
+// The stem runs as a 4x4 stride-1 convolution over the space-to-depth image
+// (2x2 pixel blocks -> 12 channels, padded to 16) with a zero border of 2
+// before and 1 after in memory: W [64, 4, 4, 16], one 64-wide k-block per
+// kernel row (4 pixels x 16 channels, contiguous in memory).
+constexpr int kS2dC = 16;
+constexpr int kStemKs = 4 * 4 * kS2dC;
 constexpr size_t kAlignB = 1024;
 
 struct BlockShape {
@@ -64,7 +69,7 @@ using F16Buf = bf16;
 
 struct CnnBlockPack {
   int a = 0, b = 0, a_pad = 0, b_pad = 0;  // kept |S_a|, |S_b| and their padded widths
-  int a_cp = 0;                            // conv2's per-tap K stride: a_pad rounded up to 64
+  int a_cp = 0;                            // conv2's per-tap K stride: conv_tap_stride(a_pad)
   F16Buf *w1 = nullptr, *w2 = nullptr, *w3 = nullptr;
   float *b1 = nullptr, *b2 = nullptr, *b3 = nullptr;
   GemmPlan conv1, conv2, conv3;
@@ -94,7 +99,7 @@ struct CnnModel {
   GemmPlan stem;
   std::vector<GemmPlan> down;  // per block (valid where the block has a projection)
   // workspace
-  F16Buf *col = nullptr, *xa = nullptr, *xb = nullptr, *t1 = nullptr, *t2 = nullptr, *sc = nullptr;
+  F16Buf *s2d = nullptr, *xa = nullptr, *xb = nullptr, *t1 = nullptr, *t2 = nullptr, *sc = nullptr;
   float* pooled = nullptr;
   void* img_stage = nullptr;
   float* logit_stage = nullptr;
@@ -150,74 +155,42 @@ __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
   return *reinterpret_cast<const uint32_t*>(&v);
 }
 
-// The stem's gather (7x7, stride 2, padding 3, 3 channels; 147 columns in
-// (ky, kx, c) order padded with zeros to 152 = 19 groups of 8).
-// One CTA per output row (image b, row oy). The seven input rows
-// the row's 7x7/2 windows cover are staged once in shared memory as f16
-// (zero outside the image, three zero columns each side), then the CTA writes
-// the Wo gathered rows [Wo, 152] ((ky, kx, c) columns, 147 padded to 152) with
-// coalesced 16-byte stores.
-constexpr int kStemWmax = 1024;  // 7 x (W + 6) x 3 f16 of shared memory: <= 43 KB
-constexpr int kStemThreads = 13 * (kStemKp / 8);  // 247: a whole number of 19-group pixels
+// Space-to-depth of the image for the stem, with its zero border:
+// S[b, 2 + y, 2 + x, (dy * 2 + dx) * 3 + c] = img[b, 2y + dy, 2x + dx, c] as
+// f16 (zero past an odd-sized image), channels 12..15 zero, S [B, Hs + 3,
+// Ws + 3, 16] zero outside y < Hs, x < Ws. One thread per S pixel (32 bytes
+// out), from the last pixel to the first: the stem GEMM reads them first to
+// last.
 template <typename T>
-__global__ void __launch_bounds__(kStemThreads) stem_im2col_kernel(const T* __restrict__ src, int H, int W, int Ho, int Wo,
-                                                          uint4* __restrict__ dst) {
+__global__ void stem_s2d_kernel(const T* __restrict__ src, int B, int H, int W, int Hs, int Ws,
+                                uint4* __restrict__ dst) {
   pdl_wait();
   pdl_trigger();
-  constexpr int G = kStemKp / 8;
-  extern __shared__ uint16_t tile_raw[];  // [ky][(ix + 3) * 3 + c], f16 bits
-  // output rows last to first: the stem GEMM reads them first to last, so the
-  // most recently written (still in L2) are the first it reads
-  const unsigned bid = gridDim.x - 1 - blockIdx.x;
-  const int oy = static_cast<int>(bid % Ho);
-  const size_t b = bid / Ho;
-  const int wp = (W + 6) * 3;
-  // eight independent loads per thread in flight before their stores
-  constexpr int U = 8;
-  for (int i0 = threadIdx.x; i0 < 7 * wp; i0 += U * blockDim.x) {
-    float v[U];
+  const int Hp = Hs + 3, Wp = Ws + 3;
+  const size_t total = static_cast<size_t>(B) * Hp * Wp;
+  for (size_t t0 = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t0 < total;
+       t0 += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const size_t t = total - 1 - t0;
+    const int x = static_cast<int>(t % Wp) - 2;
+    const size_t r = t / Wp;
+    const int y = static_cast<int>(r % Hp) - 2;
+    const size_t b = r / Hp;
+    const bool inside = y >= 0 && y < Hs && x >= 0 && x < Ws;
+    float v[16];
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + u * blockDim.x;
-      const int ky = i / wp, j = i - ky * wp;
-      const int iy = 2 * oy - 3 + ky, ix = j / 3 - 3;
-      v[u] = (i < 7 * wp && iy >= 0 && iy < H && ix >= 0 && ix < W)
-                 ? static_cast<float>(src[(b * H + iy) * W * 3 + (j - 9)])
-                 : 0.0f;
-    }
+    for (int dy = 0; dy < 2; ++dy)
 #pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const int i = i0 + u * blockDim.x;
-      if (i < 7 * wp) {
-        const __half hv = __float2half_rn(v[u]);
-        tile_raw[i] = *reinterpret_cast<const uint16_t*>(&hv);
+      for (int dx = 0; dx < 2; ++dx) {
+        const int iy = 2 * y + dy, ix = 2 * x + dx;
+        const bool in = inside && iy < H && ix < W;
+#pragma unroll
+        for (int c = 0; c < 3; ++c)
+          v[(dy * 2 + dx) * 3 + c] = in ? static_cast<float>(src[((b * H + iy) * W + ix) * 3 + c]) : 0.0f;
       }
-    }
-  }
-  __syncthreads();
-  // The CTA has 13 x 19 threads: thread T always builds column group
-  // g = T % 19 (columns 8g .. 8g + 7) of pixels ox = T / 19 + 13 i, so its
-  // eight shared-memory offsets are computed once; consecutive threads still
-  // write consecutive 16-byte pieces of the output rows.
-  const int g = threadIdx.x % G, ox0 = threadIdx.x / G;
-  int off[8];
 #pragma unroll
-  for (int e = 0; e < 8; ++e) {
-    const int k = g * 8 + e;
-    const int tap = k / 3, c = k - 3 * tap, ky = tap / 7, kx = tap - 7 * ky;
-    off[e] = k < kStemK ? ky * wp + kx * 3 + c : -1;
-  }
-  uint4* out = dst + (b * Ho + oy) * static_cast<size_t>(Wo) * G;
-  for (int ox = ox0; ox < Wo; ox += kStemThreads / G) {
-    const uint16_t* base = tile_raw + 6 * ox;
-    uint32_t u[4];
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const uint32_t lo = off[2 * q] >= 0 ? base[off[2 * q]] : 0u;
-      const uint32_t hi = off[2 * q + 1] >= 0 ? base[off[2 * q + 1]] : 0u;
-      u[q] = lo | (hi << 16);
-    }
-    out[ox * G + g] = make_uint4(u[0], u[1], u[2], u[3]);
+    for (int c = 12; c < 16; ++c) v[c] = 0.0f;
+    dst[2 * t] = make_uint4(pack2(v[0], v[1]), pack2(v[2], v[3]), pack2(v[4], v[5]), pack2(v[6], v[7]));
+    dst[2 * t + 1] = make_uint4(pack2(v[8], v[9]), pack2(v[10], v[11]), pack2(v[12], v[13]), pack2(v[14], v[15]));
   }
 }
 
@@ -339,18 +312,16 @@ unsigned grid_for(size_t n) {
   return static_cast<unsigned>(b < 16384 ? (b > 0 ? b : 1) : 16384);
 }
 
-cudaError_t stem_im2col_launch(const void* images, int dtype, int B, int H, int W, int Ho, int Wo, __half* dst,
-                               cudaStream_t s) {
-  if (B <= 0 || Ho <= 0 || Wo <= 0) return cudaSuccess;
-  if (W > kStemWmax) return cudaErrorInvalidValue;
-  const unsigned blocks = static_cast<unsigned>(B) * Ho;
-  const size_t smem = size_t(7) * (W + 6) * 3 * 2;
+cudaError_t stem_s2d_launch(const void* images, int dtype, int B, int H, int W, int Hs, int Ws, __half* dst,
+                            cudaStream_t s) {
+  const size_t total = static_cast<size_t>(B) * (Hs + 3) * (Ws + 3);
+  if (total == 0) return cudaSuccess;
   uint4* d = reinterpret_cast<uint4*>(dst);
   if (dtype == ELASTO_BF16)
-    return launch_pdl(stem_im2col_kernel<bf16>, dim3(blocks), dim3(kStemThreads), smem, s,
-                      static_cast<const bf16*>(images), H, W, Ho, Wo, d);
-  return launch_pdl(stem_im2col_kernel<float>, dim3(blocks), dim3(kStemThreads), smem, s,
-                    static_cast<const float*>(images), H, W, Ho, Wo, d);
+    return launch_pdl(stem_s2d_kernel<bf16>, dim3(grid_for(total)), dim3(256), 0, s, static_cast<const bf16*>(images),
+                      B, H, W, Hs, Ws, d);
+  return launch_pdl(stem_s2d_kernel<float>, dim3(grid_for(total)), dim3(256), 0, s, static_cast<const float*>(images),
+                    B, H, W, Hs, Ws, d);
 }
 
 // ---------------------------------------------------------------- host packing
@@ -493,7 +464,7 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
 
   // ---------------------------------------------------------------- layout
   Arena ar;
-  const size_t o_stem_w = ar.take(size_t(kStemC) * kStemKp * 2), o_stem_b = ar.take(kStemC * 4);
+  const size_t o_stem_w = ar.take(size_t(kStemC) * kStemKs * 2), o_stem_b = ar.take(kStemC * 4);
   std::vector<size_t> o_dw(nblk, 0), o_db(nblk, 0);
   for (int i = 0; i < nblk; ++i)
     if (S[i].proj) {
@@ -517,7 +488,7 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
         bp.b = tables[mo].n_conv_b[i];
         bp.a_pad = round8(bp.a);
         bp.b_pad = round8(bp.b);
-        bp.a_cp = (bp.a_pad + 63) / 64 * 64;
+        bp.a_cp = conv_tap_stride(bp.a_pad);
         Off& o = offs[mo][i];
         o.w1 = ar.take(size_t(bp.a_pad) * S[i].cin * 2);
         o.b1 = ar.take(size_t(bp.a_pad) * 4);
@@ -531,7 +502,8 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
   }
   // workspace (sizes for the widest mode: kept counts never exceed the width)
   const size_t rows_stem = size_t(Bm) * m->h1 * m->w1;
-  const size_t col = rows_stem * kStemKp;  // only the stem is gathered
+  // the space-to-depth image with its border: (stem output size + 3)^2 x 16
+  const size_t s2d = size_t(Bm) * (m->h1 + 3) * (m->w1 + 3) * kS2dC;
   size_t xbuf = std::max(rows_stem * kStemC, size_t(Bm) * m->hp * m->wp * kStemC);
   size_t t1 = 0, t2 = 0, scb = 0;
   for (const BlockShape& b : S) {
@@ -542,7 +514,7 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
     if (b.proj) scb = std::max(scb, ro * 4 * size_t(b.w));
   }
   const size_t ws_start = ar.off;
-  const size_t o_col = ar.take(col * 2), o_xa = ar.take(xbuf * 2), o_xb = ar.take(xbuf * 2);
+  const size_t o_s2d = ar.take(s2d * 2), o_xa = ar.take(xbuf * 2), o_xb = ar.take(xbuf * 2);
   const size_t o_t1 = ar.take(t1 * 2), o_t2 = ar.take(t2 * 2), o_sc = ar.take(scb * 2);
   const size_t o_pool = ar.take(size_t(Bm) * 2048 * 4);
   const size_t o_img = ar.take(size_t(Bm) * d->img_h * d->img_w * 3 * (dt == ELASTO_BF16 ? 2 : 4));
@@ -571,7 +543,7 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
     }
   m->fc_w = reinterpret_cast<float*>(A + o_fcw);
   m->fc_b = reinterpret_cast<float*>(A + o_fcb);
-  m->col = reinterpret_cast<F16Buf*>(A + o_col);
+  m->s2d = reinterpret_cast<F16Buf*>(A + o_s2d);
   m->xa = reinterpret_cast<F16Buf*>(A + o_xa);
   m->xb = reinterpret_cast<F16Buf*>(A + o_xb);
   m->t1 = reinterpret_cast<F16Buf*>(A + o_t1);
@@ -598,18 +570,25 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
   std::vector<float> hb;
   auto up16 = [&](void* dst) { return cudaMemcpy(dst, hw.data(), hw.size() * 2, cudaMemcpyHostToDevice); };
   auto up32 = [&](void* dst) { return cudaMemcpy(dst, hb.data(), hb.size() * 4, cudaMemcpyHostToDevice); };
-  {  // stem: [64, (ky, kx, c) padded to 152] from [64, 3, 7, 7]
+  {  // stem: [64, 4, 4, 16] over the space-to-depth image from [64, 3, 7, 7]: tap (ty, tx)
+     // reads S rows y - 2 + ty, i.e. image rows 2y - 4 + 2 ty + dy = 2y - 3 + ky with
+     // ky = 2 ty + dy - 1 (likewise kx); taps outside 0..6 stay zero
     const HostTensor W = T(t_stem);
     const Bn bn{T(t_stem + 1), T(t_stem + 2), T(t_stem + 3), T(t_stem + 4)};
-    hw.assign(size_t(kStemC) * kStemKp, 0);
+    hw.assign(size_t(kStemC) * kStemKs, 0);
     hb.assign(kStemC, 0.0f);
     for (int o = 0; o < kStemC; ++o) {
       const double s = bn.scale(o);
-      for (int c = 0; c < 3; ++c)
-        for (int ky = 0; ky < 7; ++ky)
-          for (int kx = 0; kx < 7; ++kx)
-            hw[size_t(o) * kStemKp + (ky * 7 + kx) * 3 + c] =
-                f16_bits(static_cast<float>(W[((size_t(o) * 3 + c) * 7 + ky) * 7 + kx] * s));
+      for (int ty = 0; ty < 4; ++ty)
+        for (int tx = 0; tx < 4; ++tx)
+          for (int dy = 0; dy < 2; ++dy)
+            for (int dx = 0; dx < 2; ++dx) {
+              const int ky = 2 * ty + dy - 1, kx = 2 * tx + dx - 1;
+              if (ky < 0 || ky > 6 || kx < 0 || kx > 6) continue;
+              for (int c = 0; c < 3; ++c)
+                hw[size_t(o) * kStemKs + (ty * 4 + tx) * kS2dC + (dy * 2 + dx) * 3 + c] =
+                    f16_bits(static_cast<float>(W[((size_t(o) * 3 + c) * 7 + ky) * 7 + kx] * s));
+            }
       hb[o] = static_cast<float>(bn.bias(o));
     }
     ELASTO_CUDA_TRY(up16(m->stem_w));
@@ -694,8 +673,10 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
   }
 
   // ---------------------------------------------------------------- plans
-  elasto_status st = gemm_plan(&m->stem, m->col, int(rows_stem), m->stem_w, kStemC, kStemKp, m->stem_b, m->xb,
-                                  kStemC, EPI_BIAS_RELU_F16, m->status);
+  // the stem: 4x4 stride-1 convolution over the bordered space-to-depth image
+  // ((h1 + 3) x (w1 + 3) x 16), output h1 x w1 (the 7x7/2 convolution's)
+  elasto_status st = gemm_plan_conv_rows(&m->stem, m->s2d, Bm, m->h1 + 3, m->w1 + 3, kS2dC, 4, 4, m->stem_w, kStemC,
+                                         m->stem_b, m->xb, kStemC, EPI_BIAS_RELU_F16, m->status);
   if (st != ELASTO_OK) return st;
   m->down.assign(nblk, GemmPlan{});
   const int64_t stem_macs = int64_t(m->h1) * m->w1 * kStemC * kStemK + int64_t(2048) * C;
@@ -760,11 +741,11 @@ elasto_status cnn_forward(CnnModel* m, int mode, cudaStream_t s, const void* ima
   const double img_elt = d.weight_dtype == ELASTO_BF16 ? 2 : 4;
   m->prof.begin();
   const int ms = B * m->h1 * m->w1;
-  CNN_LAUNCH(rec(ELASTO_K_IM2COL, -1, ms, kStemKp, 0, 0,
-                 double(B) * d.img_h * d.img_w * 3 * img_elt + double(ms) * kStemKp * 2),
-             stem_im2col_launch(images, d.weight_dtype, B, d.img_h, d.img_w, m->h1, m->w1,
-                                reinterpret_cast<__half*>(m->col), s));
-  CNN_LAUNCH(gemm_record(-1, ms, kStemC, kStemK, false), gemm_launch(m->stem, ms, s));
+  CNN_LAUNCH(rec(ELASTO_K_IM2COL, -1, ms, kS2dC, 0, 0,
+                 double(B) * d.img_h * d.img_w * 3 * img_elt + double(B) * (m->h1 + 3) * (m->w1 + 3) * kS2dC * 2),
+             stem_s2d_launch(images, d.weight_dtype, B, d.img_h, d.img_w, m->h1, m->w1,
+                             reinterpret_cast<__half*>(m->s2d), s));
+  CNN_LAUNCH(gemm_record(-1, ms, kStemC, kStemK, false), gemm_launch(m->stem, B, s));
   {
     const size_t total = size_t(B) * m->hp * m->wp * (kStemC / 8);
     CNN_LAUNCH(rec(ELASTO_K_POOL, -1, B * m->hp * m->wp, kStemC, 0, 0,

@@ -64,8 +64,13 @@ bool encode_tmap_2d(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t 
 // 4-D f16 tensor (NHWC activations: dims {C, W, H, B}), byte strides of
 // dims 1..3, box in traversed elements, traversal strides (the box loads
 // ceil(box[i] / elem_strides[i]) elements along dim i), 128-byte swizzle.
+// 16-bit f16 4-D map (NHWC activations), 128-byte swizzle, or 32-byte when
+// sw32 (16-channel boxes: one 32-byte row per pixel).
 bool encode_tmap_4d(CUtensorMap* tm, const void* base, const uint64_t dims[4], const uint64_t strides_bytes[3],
-                    const uint32_t box[4], const uint32_t elem_strides[4]);
+                    const uint32_t box[4], const uint32_t elem_strides[4], bool sw32 = false);
+// 16-bit f16 2-D map with the 32-byte swizzle.
+bool encode_tmap_2d_sw32(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_stride_bytes,
+                         uint32_t box_inner, uint32_t box_outer);
 // 3-D bf16 tensor [d2][d1][d0] with byte strides s1 (between d1 rows) and s2.
 bool encode_tmap_3d(CUtensorMap* tm, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1,
                     uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2);
@@ -112,6 +117,8 @@ struct GemmArgs {
   int cv_a_bytes;                            // bytes one A tile load delivers
   int resid_row_mod;                         // > 0: periodic residual source (gemm_set_residual_source)
   int m_reverse;                             // 1: tile rows scheduled last to first (L2 reuse of A)
+  int k16;                                   // implicit conv on <= 16 channels: k-blocks of 16 (one tap each),
+                                             // operands in the 32-byte swizzle
 };
 
 struct GemmPlan {
@@ -158,12 +165,28 @@ struct GemmPlanSet {
 // M_cap >= row_period + 128 of them; output row r adds src row r mod period
 // (a tile starting at m0 reads rows m0 mod period ... + 127).
 elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap, int row_period = 0);
+// Per-tap K stride of an implicit-GEMM convolution's weights: 16 for up to 16
+// channels (one 16-wide k-block per tap, 32-byte swizzle), else C rounded up
+// to 64 (64-channel k-blocks).
+inline int conv_tap_stride(int C) { return C <= 16 ? 16 : (C + 63) / 64 * 64; }
 // Implicit-GEMM k x k convolution (stride, padding `pad`) of the f16 NHWC
-// input x [B_cap, H, W, C] (C % 8 == 0) with W [N, k * k * Cp] f16, Cp = C
-// rounded up to 64 (zero columns), out = epi(conv + bias) f16 [B_cap, Ho, Wo,
-// ldo] (EPI_BIAS_RELU_F16 or EPI_BIAS_F16). gemm_launch's M is the batch.
+// input x [B_cap, H, W, C] (C % 8 == 0) with W [N, k * k * conv_tap_stride(C)]
+// f16 (each tap's channels zero-padded), out = epi(conv + bias) f16 [B_cap,
+// Ho, Wo, ldo] (EPI_BIAS_RELU_F16 or EPI_BIAS_F16). gemm_launch's M is the
+// batch.
+// Ho_out / Wo_out > 0 replace the output size (a smaller output window).
 elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W, int C, int k, int stride, int pad,
-                             const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status);
+                             const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status,
+                             int Ho_out = 0, int Wo_out = 0);
+// Stride-1 convolution without padding of an input already padded in memory,
+// x [B_cap, Hp, Wp, C] f16, whose kernel rows are kw * C == 64 contiguous
+// values: kernel row ky of output pixel (y, x) reads x[b, y + ky, x .. x + kw
+// - 1, :], which is one 64-wide k-block. W [N, kh * kw * C] f16 in (ky, kx,
+// c) order; out as for gemm_plan_conv, over Ho = Hp - kh + 1, Wo = Wp - kw + 1
+// or the smaller window Ho_out x Wo_out.
+elasto_status gemm_plan_conv_rows(GemmPlan* p, const void* x, int B_cap, int Hp, int Wp, int C, int kh, int kw,
+                                  const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status,
+                                  int Ho_out = 0, int Wo_out = 0);
 // Launch for the first M (<= M_cap) rows.
 cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s);
 cudaError_t gemm_init_attributes();

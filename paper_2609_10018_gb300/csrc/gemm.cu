@@ -204,7 +204,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int M = args.M, N = args.N, bn = args.bn;
-  const int nk = (args.K + BK - 1) / BK;
+  const int bke = args.k16 ? 16 : BK;  // K values per k-block
+  const int nk = (args.K + bke - 1) / bke;
   constexpr int TM = PAIR ? 2 * BM : BM;  // rows per tile
   const int mt = args.conv ? conv_mtiles(args) : (M + TM - 1) / TM, nt = (N + bn - 1) / bn;
   const int tiles = mt * nt;
@@ -263,7 +264,7 @@ __global__ void __launch_bounds__(THREADS, 1)
       bool ok = true;
       // pair: the even CTA's full barrier counts both CTAs' bytes
       const uint32_t bytes =
-          PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2) : (args.conv ? args.cv_a_bytes : A_STAGE) + NB * bn * BK * 2;
+          PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2) : (args.conv ? args.cv_a_bytes : A_STAGE) + NB * bn * bke * 2;
       for (int t = t_start; t < tiles && ok; t += t_stride) {
         const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
         int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
@@ -289,12 +290,12 @@ __global__ void __launch_bounds__(THREADS, 1)
           if (args.conv) {
             const int tap = kb / args.cv_cgroups, cg = kb - tap * args.cv_cgroups;
             const int ky = tap / args.cv_ks, kx = tap - ky * args.cv_ks;
-            tma_load_4d(sA + stage * A_STAGE, &tmA, &full[stage], cg * BK, cx0 * args.cv_stride - args.cv_pad + kx,
+            tma_load_4d(sA + stage * A_STAGE, &tmA, &full[stage], cg * bke, cx0 * args.cv_stride - args.cv_pad + kx,
                         cy0 * args.cv_stride - args.cv_pad + ky, cb0);
           } else {
             tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
           }
-          tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * BK, n0);
+          tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * bke, n0);
           if constexpr (NB == 2) tma_load_2d(sB + stage * BSTG + BSTG / 2, &tmB2, &full[stage], kb * BK, n0);
           ++issued;
           if (++stage == S) {
@@ -346,6 +347,12 @@ __global__ void __launch_bounds__(THREADS, 1)
           }
           tc_fence_after();
           const uint32_t a0 = smem_addr(sA + stage * A_STAGE), b0 = smem_addr(sB + stage * BSTG);
+          if (args.k16) {
+            // one K=16 step per k-block: rows of 32 bytes in the 32-byte swizzle,
+            // 8-row groups 256 bytes apart
+            if constexpr (!PAIR && NB == 1)
+              tc_mma(dtm, sdesc_sw32(a0, 16, 256), sdesc_sw32(b0, 16, 256), idesc, kb != 0);
+          } else
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             if constexpr (PAIR) {
@@ -823,26 +830,25 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   return ELASTO_OK;
 }
 
-elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W, int C, int k, int stride, int pad,
-                             const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status) {
-  if (!p || !x || !Wt || !out || B_cap <= 0 || H <= 0 || W <= 0 || C <= 0 || k <= 0 || stride <= 0 || pad < 0 ||
-      N <= 0 || (epi != EPI_BIAS_RELU_F16 && epi != EPI_BIAS_F16)) {
-    set_error("gemm_plan_conv: invalid arguments");
-    return ELASTO_ERR_INVALID_ARG;
-  }
-  const int Ho = (H + 2 * pad - k) / stride + 1, Wo = (W + 2 * pad - k) / stride + 1;
-  if (C % 8 != 0 || ldo % 8 != 0 || N % 2 != 0 || N > ldo || Ho <= 0 || Wo <= 0 || stride > 2) {
-    set_error("gemm_plan_conv: needs C and ldo multiples of 8, N even, stride 1 or 2");
-    return ELASTO_ERR_UNSUPPORTED;
-  }
+namespace {
+
+// The part both convolution plans share. A is read through the 4D map
+// {channels, x, y, image} = xd (byte strides xs) in boxes of bke channels by
+// the tile's pixel block; k-block kb covers tap kb / cg (ky = tap / taps_x,
+// kx = tap % taps_x) and channel group kb % cg.
+elasto_status plan_conv_common(GemmPlan* p, const char* who, const void* x, const uint64_t xd[4],
+                               const uint64_t xs[3], int B_cap, int Ho, int Wo, int taps, int taps_x, int cg, int bke,
+                               int stride, int pad, const void* Wt, int N, const float* bias, void* out, int ldo,
+                               int epi, int* status) {
   *p = GemmPlan{};
   GemmArgs& a = p->args;
-  const int cg = (C + BK - 1) / BK;
+  const bool k16 = bke == 16;
   a.M = B_cap;
   a.N = N;
-  a.K = k * k * cg * BK;
+  a.K = taps * cg * bke;
+  a.k16 = k16 ? 1 : 0;
   a.conv = 1;
-  a.cv_ks = k;
+  a.cv_ks = taps_x;
   a.cv_stride = stride;
   a.cv_pad = pad;
   a.cv_cgroups = cg;
@@ -868,7 +874,7 @@ elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W
       }
     }
   const int rows = a.cv_bw * a.cv_bh * a.cv_nb;
-  a.cv_a_bytes = rows * BK * 2;
+  a.cv_a_bytes = rows * bke * 2;
   a.cv_batch = B_cap;
   a.bn = gemm_pick_bn(conv_mtiles(a) * BM, N, 64, false);
   a.bias = bias;
@@ -884,26 +890,86 @@ elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W
   a.cbufs = (POOL - a.stages * (A_STAGE + a.b_stage)) / CBUF;
   if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
   if (a.cbufs < 2 || rows > BM || a.stages < 2) {
-    set_error("gemm_plan_conv: shared-memory layout does not fit");
+    set_error(std::string(who) + ": shared-memory layout does not fit");
     return ELASTO_ERR_UNSUPPORTED;
   }
-  const uint64_t xd[4] = {uint64_t(C), uint64_t(W), uint64_t(H), uint64_t(B_cap)};
-  const uint64_t xs[3] = {uint64_t(C) * 2, uint64_t(W) * C * 2, uint64_t(H) * W * C * 2};
-  const uint32_t xb[4] = {uint32_t(BK), uint32_t(a.cv_bw * stride), uint32_t(a.cv_bh * stride), uint32_t(a.cv_nb)};
+  const uint32_t xb[4] = {uint32_t(bke), uint32_t(a.cv_bw * stride), uint32_t(a.cv_bh * stride), uint32_t(a.cv_nb)};
   const uint32_t xe[4] = {1u, uint32_t(stride), uint32_t(stride), 1u};
   const uint64_t od[4] = {uint64_t(N), uint64_t(Wo), uint64_t(Ho), uint64_t(B_cap)};
   const uint64_t os[3] = {uint64_t(ldo) * 2, uint64_t(Wo) * ldo * 2, uint64_t(Ho) * Wo * ldo * 2};
   const uint32_t ob[4] = {64u, uint32_t(a.cv_bw), uint32_t(a.cv_bh), uint32_t(a.cv_nb)};
   const uint32_t oe[4] = {1u, 1u, 1u, 1u};
-  if (xb[1] > 256 || xb[2] > 256 || !encode_tmap_4d(&p->tmA, x, xd, xs, xb, xe) ||
-      !encode_tmap_2d(&p->tmB, Wt, a.K, N, uint64_t(a.K) * 2, BK, a.bn) || !encode_tmap_4d(&p->tmC, out, od, os, ob, oe)) {
-    set_error("gemm_plan_conv: cuTensorMapEncodeTiled failed (alignment or size)");
+  const bool wmap = k16 ? encode_tmap_2d_sw32(&p->tmB, Wt, a.K, N, uint64_t(a.K) * 2, 16, a.bn)
+                        : encode_tmap_2d(&p->tmB, Wt, a.K, N, uint64_t(a.K) * 2, BK, a.bn);
+  if (xb[1] > 256 || xb[2] > 256 || !encode_tmap_4d(&p->tmA, x, xd, xs, xb, xe, k16) || !wmap ||
+      !encode_tmap_4d(&p->tmC, out, od, os, ob, oe)) {
+    set_error(std::string(who) + ": cuTensorMapEncodeTiled failed (alignment or size)");
     return ELASTO_ERR_UNSUPPORTED;
   }
   p->tmR = p->tmC;
   p->epi = epi;
   p->valid = true;
   return ELASTO_OK;
+}
+
+bool conv_args_ok(const GemmPlan* p, const void* x, const void* Wt, void* out, int B_cap, int N, int ldo, int epi) {
+  return p && x && Wt && out && B_cap > 0 && N > 0 && (epi == EPI_BIAS_RELU_F16 || epi == EPI_BIAS_F16);
+}
+
+}  // namespace
+
+elasto_status gemm_plan_conv(GemmPlan* p, const void* x, int B_cap, int H, int W, int C, int k, int stride, int pad,
+                             const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status,
+                             int Ho_out, int Wo_out) {
+  if (!conv_args_ok(p, x, Wt, out, B_cap, N, ldo, epi) || H <= 0 || W <= 0 || C <= 0 || k <= 0 || stride <= 0 ||
+      pad < 0) {
+    set_error("gemm_plan_conv: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int Ho_full = (H + 2 * pad - k) / stride + 1, Wo_full = (W + 2 * pad - k) / stride + 1;
+  const int Ho = Ho_out > 0 ? Ho_out : Ho_full, Wo = Wo_out > 0 ? Wo_out : Wo_full;
+  if (Ho > Ho_full || Wo > Wo_full) {
+    set_error("gemm_plan_conv: the output window exceeds the convolution's output");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (C % 8 != 0 || ldo % 8 != 0 || N % 2 != 0 || N > ldo || Ho <= 0 || Wo <= 0 || stride > 2) {
+    set_error("gemm_plan_conv: needs C and ldo multiples of 8, N even, stride 1 or 2");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  // up to 16 channels: one 16-wide k-block per tap (32-byte swizzle) instead
+  // of a 64-channel group that would be three quarters zeros
+  const int bke = conv_tap_stride(C) == 16 ? 16 : BK;
+  const uint64_t xd[4] = {uint64_t(C), uint64_t(W), uint64_t(H), uint64_t(B_cap)};
+  const uint64_t xs[3] = {uint64_t(C) * 2, uint64_t(W) * C * 2, uint64_t(H) * W * C * 2};
+  return plan_conv_common(p, "gemm_plan_conv", x, xd, xs, B_cap, Ho, Wo, k * k, k, conv_tap_stride(C) / bke, bke,
+                          stride, pad, Wt, N, bias, out, ldo, epi, status);
+}
+
+elasto_status gemm_plan_conv_rows(GemmPlan* p, const void* x, int B_cap, int Hp, int Wp, int C, int kh, int kw,
+                                  const void* Wt, int N, const float* bias, void* out, int ldo, int epi, int* status,
+                                  int Ho_out, int Wo_out) {
+  if (!conv_args_ok(p, x, Wt, out, B_cap, N, ldo, epi) || C <= 0 || kh <= 0 || kw <= 0 || Hp < kh || Wp < kw) {
+    set_error("gemm_plan_conv_rows: invalid arguments");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  const int Ho_full = Hp - kh + 1, Wo_full = Wp - kw + 1;
+  const int Ho = Ho_out > 0 ? Ho_out : Ho_full, Wo = Wo_out > 0 ? Wo_out : Wo_full;
+  if (Ho > Ho_full || Wo > Wo_full) {
+    set_error("gemm_plan_conv_rows: the output window exceeds the convolution's output");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (kw * C != BK || C % 8 != 0 || ldo % 8 != 0 || N % 2 != 0 || N > ldo) {
+    set_error("gemm_plan_conv_rows: needs kw * C == 64, C and ldo multiples of 8, N even");
+    return ELASTO_ERR_UNSUPPORTED;
+  }
+  // the map's x axis steps one pixel (C channels) while each box row takes
+  // kw * C = 64 values: the kw pixels that kernel row ky meets, overlapping
+  // the next row's; x runs over the Wo_full window starts only, so no box row
+  // reaches past the end of an input row
+  const uint64_t xd[4] = {uint64_t(BK), uint64_t(Wo_full), uint64_t(Hp), uint64_t(B_cap)};
+  const uint64_t xs[3] = {uint64_t(C) * 2, uint64_t(Wp) * C * 2, uint64_t(Hp) * Wp * C * 2};
+  return plan_conv_common(p, "gemm_plan_conv_rows", x, xd, xs, B_cap, Ho, Wo, kh, 1, 1, BK, 1, 0, Wt, N, bias, out,
+                          ldo, epi, status);
 }
 
 elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap, int row_period) {

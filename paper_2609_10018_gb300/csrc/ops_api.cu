@@ -91,9 +91,8 @@ elasto_status elasto_op_layernorm(void* stream, const float* x, const float* gam
     set_error("elasto_op_layernorm: invalid arguments");
     return ELASTO_ERR_INVALID_ARG;
   }
-  const int v = d / 64;
-  if (d % 64 != 0 || !(v <= 6 || v == 8 || v == 10 || v == 12 || v == 16)) {
-    set_error("elasto_op_layernorm: d must be 64 x {1..6, 8, 10, 12, 16}");
+  if (d % 64 != 0 || d > 1024) {
+    set_error("elasto_op_layernorm: d must be a multiple of 64 up to 1024");
     return ELASTO_ERR_UNSUPPORTED;
   }
   ELASTO_CUDA_TRY(

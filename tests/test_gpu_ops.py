@@ -224,7 +224,9 @@ CONV_CASES = [
     (5, 7, 7, 136, 48, 1, 2, 0, False),      # strided 1x1 projection, 3 channel groups (ragged)
     (1, 56, 56, 64, 64, 3, 1, 1, True),      # ResNet-50 stage 1 conv2 at batch 1
     (40, 2, 2, 512, 512, 3, 1, 1, True),     # whole images per tile (nb > 1)
-    (4, 9, 9, 16, 24, 3, 2, 1, False),       # N below one 64-column chunk, stride 2
+    (4, 9, 9, 16, 24, 3, 2, 1, False),       # N below one 64-column chunk, stride 2 (16-channel k-blocks)
+    (3, 11, 13, 8, 40, 3, 1, 1, True),       # 8 channels: 16-wide k-blocks, half of each zero
+    (2, 20, 20, 16, 64, 4, 1, 2, True),      # 4 x 4 taps on 16 channels (the space-to-depth stem's shape)
 ]
 
 
@@ -236,7 +238,7 @@ def test_conv2d_implicit_gemm_matches_fp64(B, H, W, C, N, k, stride, pad, relu):
     x = _f16(rng, (B, H, W, C))
     wt = (rng.standard_normal((N, C, k, k)) * np.sqrt(2.0 / (C * k * k))).astype(np.float16)
     bias = rng.standard_normal(N).astype(np.float32) * 0.1
-    cp = (C + 63) // 64 * 64
+    cp = 16 if C <= 16 else (C + 63) // 64 * 64
     packed = np.zeros((N, k, k, cp), np.float16)
     packed[..., :C] = wt.transpose(0, 2, 3, 1)
     ref = orr.conv2d(_f16_to_f64(x), wt.astype(np.float64), stride, pad) + bias

@@ -129,6 +129,22 @@ def test_resnet_batch_1_and_ragged_and_switch():
             assert np.array_equal(_run(model, x7, 7, cfg.classes, m), first[m])
 
 
+@pytest.mark.parametrize("img_size", [45, 34])
+def test_resnet_odd_and_even_image_sizes(img_size):
+    """The stem at sizes other than 32 and 224: 45 is odd (the last 2x2 pixel
+    block of the space-to-depth image is half outside the image), 34 gives a
+    stem output of 17 (odd, so no pixel block tiles it evenly)."""
+    cfg = dataclasses.replace(SMALL, name=f"resnet50_{img_size}px", img=img_size)
+    w, tables = synth.make_resnet_weights(cfg), synth.make_resnet_tables(cfg)
+    img = synth.make_images(cfg, 9, seed=11)
+    with binding.ElasticModel.resnet(cfg, w, tables, max_batch=9) as model:
+        x = dev(img)
+        for m in (0, cfg.n_modes - 1):
+            got, ref = _run(model, x, 9, cfg.classes, m), resnet_logits(cfg, tables, m, img)
+            _report(f"resnet50 {img_size}px mode {m}", got, ref)
+            assert rel_err(got, ref) <= TOL
+
+
 def test_resnet_kept_counts_not_multiple_of_8():
     """Kept sets of 5, 13, 27 ... channels (zero-padded inside the library)."""
     cfg = SMALL
