@@ -64,6 +64,7 @@ cudaError_t ensure_kernel_attributes() {
   std::call_once(g_attr_once[dev], [dev] {
     cudaError_t r = gemm_init_attributes();
     if (r == cudaSuccess) r = attn_init_attributes();
+    if (r == cudaSuccess) r = cnn_init_attributes();
     g_attr_err[dev] = r;
   });
   return g_attr_err[dev];

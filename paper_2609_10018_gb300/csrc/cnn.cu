@@ -214,9 +214,11 @@ __global__ void maxpool_kernel(const uint4* __restrict__ src, int H, int W, int 
     float m[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) m[j] = -INFINITY;
+#pragma unroll
     for (int ky = 0; ky < 3; ++ky) {
       const int iy = 2 * oy - 1 + ky;
       if (iy < 0 || iy >= H) continue;
+#pragma unroll
       for (int kx = 0; kx < 3; ++kx) {
         const int ix = 2 * ox - 1 + kx;
         if (ix < 0 || ix >= W) continue;
@@ -240,6 +242,7 @@ __global__ void avgpool_kernel(const uint4* __restrict__ src, int HW, int C8, si
     const int c8 = static_cast<int>(t % C8);
     const size_t b = t / C8;
     float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 7
     for (int p = 0; p < HW; ++p) {
       float f[8];
       unpack8(src[(b * HW + p) * C8 + c8], f);
@@ -262,40 +265,48 @@ __device__ __forceinline__ float warp_sum32(float v) {
 constexpr int FC_IMGS = 8, FC_CPW = 4, FC_CLASSES = 8 * FC_CPW;
 
 // logits[b, c] = pooled[b, :] . Wf[c, :] + bf[c] in fp32. grid (ceil(B / 8),
-// ceil(C / 32)), 256 threads: each warp computes 4 classes x 8 images at once,
-// so every pooled float4 it loads feeds 16 FMAs and every classifier float4
-// 32 (the pooled rows are read from L1 once per 4 classes, not per class).
+// ceil(C / 32)), 256 threads: the CTA first copies its 8 pooled rows into
+// shared memory (zeros past the batch), then each warp computes 4 classes x 8
+// images at once: every classifier float4 it loads feeds 32 FMAs and the
+// pooled values come from shared memory, so the only global loads in the loop
+// are the four independent classifier rows.
 __global__ void __launch_bounds__(256) fc_kernel(const float* __restrict__ pooled, int B, int d,
                                                  const float* __restrict__ Wf, const float* __restrict__ bf, int C,
                                                  float* __restrict__ logits) {
   pdl_wait();
   pdl_trigger();
+  extern __shared__ float4 sy4[];  // [FC_IMGS][d / 4]
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int b0 = blockIdx.x * FC_IMGS;
   const int nimg = min(FC_IMGS, B - b0);
+  const int d4 = d / 4;
+  for (int t = threadIdx.x; t < FC_IMGS * d4; t += blockDim.x) {
+    const int i = t / d4;
+    sy4[t] = i < nimg ? reinterpret_cast<const float4*>(pooled + static_cast<size_t>(b0 + i) * d)[t - i * d4]
+                      : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncthreads();
   const int c0 = blockIdx.y * FC_CLASSES + warp * FC_CPW;
   if (c0 >= C) return;
-  const float* wr[FC_CPW];
+  const float4* wr[FC_CPW];
 #pragma unroll
-  for (int j = 0; j < FC_CPW; ++j) wr[j] = Wf + static_cast<size_t>(min(c0 + j, C - 1)) * d;
+  for (int j = 0; j < FC_CPW; ++j) wr[j] = reinterpret_cast<const float4*>(Wf + static_cast<size_t>(min(c0 + j, C - 1)) * d);
   float acc[FC_CPW][FC_IMGS];
 #pragma unroll
   for (int j = 0; j < FC_CPW; ++j)
 #pragma unroll
     for (int i = 0; i < FC_IMGS; ++i) acc[j][i] = 0.0f;
-#pragma unroll 2
-  for (int c = lane * 4; c < d; c += 128) {
+#pragma unroll 4
+  for (int c = lane; c < d4; c += 32) {
     float4 wv[FC_CPW];
 #pragma unroll
-    for (int j = 0; j < FC_CPW; ++j) wv[j] = *reinterpret_cast<const float4*>(wr[j] + c);
+    for (int j = 0; j < FC_CPW; ++j) wv[j] = wr[j][c];
 #pragma unroll
     for (int i = 0; i < FC_IMGS; ++i) {
-      if (i < nimg) {
-        const float4 yv = *reinterpret_cast<const float4*>(pooled + static_cast<size_t>(b0 + i) * d + c);
+      const float4 yv = sy4[i * d4 + c];
 #pragma unroll
-        for (int j = 0; j < FC_CPW; ++j)
-          acc[j][i] += wv[j].x * yv.x + wv[j].y * yv.y + wv[j].z * yv.z + wv[j].w * yv.w;
-      }
+      for (int j = 0; j < FC_CPW; ++j)
+        acc[j][i] += wv[j].x * yv.x + wv[j].y * yv.y + wv[j].z * yv.z + wv[j].w * yv.w;
     }
   }
 #pragma unroll
@@ -306,6 +317,15 @@ __global__ void __launch_bounds__(256) fc_kernel(const float* __restrict__ poole
       if (lane == 0 && i < nimg && c0 + j < C) logits[static_cast<size_t>(b0 + i) * C + c0 + j] = v + bf[c0 + j];
     }
 }
+
+}  // namespace
+
+cudaError_t cnn_init_attributes() {
+  return cudaFuncSetAttribute(fc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              FC_IMGS * kCnnMaxFeatures * static_cast<int>(sizeof(float)));
+}
+
+namespace {
 
 unsigned grid_for(size_t n) {
   const size_t b = (n + 255) / 256;
@@ -778,10 +798,12 @@ elasto_status cnn_forward(CnnModel* m, int mode, cudaStream_t s, const void* ima
                           hw, cfin / 8, total, m->pooled));
   }
   {
+    static_assert(4 * 512 <= kCnnMaxFeatures, "the classifier's pooled rows exceed its shared-memory limit");
     dim3 grid((B + FC_IMGS - 1) / FC_IMGS, (C + FC_CLASSES - 1) / FC_CLASSES);
     CNN_LAUNCH(rec(ELASTO_K_HEAD, -1, B, C, cfin, double(B) * C * cfin,
                    double(B) * cfin * 4 + double(C) * cfin * 4 + double(B) * C * 4),
-               launch_pdl(fc_kernel, grid, dim3(256), 0, s, static_cast<const float*>(m->pooled), B, cfin,
+               launch_pdl(fc_kernel, grid, dim3(256), FC_IMGS * cfin * sizeof(float), s,
+                          static_cast<const float*>(m->pooled), B, cfin,
                           static_cast<const float*>(m->fc_w), static_cast<const float*>(m->fc_b), C, logits));
   }
   return ELASTO_OK;

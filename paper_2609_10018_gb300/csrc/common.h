@@ -119,6 +119,8 @@ struct GemmArgs {
   int m_reverse;                             // 1: tile rows scheduled last to first (L2 reuse of A)
   int k16;                                   // implicit conv on <= 16 channels: k-blocks of 16 (one tap each),
                                              // operands in the 32-byte swizzle
+  int b_resident;                            // 1: all of W (one N tile) is loaded once per CTA and kept in
+                                             // shared memory; the ring carries A only
 };
 
 struct GemmPlan {
@@ -206,6 +208,10 @@ elasto_status attn_plan(AttnPlan* p, const bf16* qkv, bf16* out, int batch_cap, 
                         bool interleaved = false);
 cudaError_t attn_launch(const AttnPlan& p, int batch, cudaStream_t s);
 cudaError_t attn_init_attributes();
+// The CNN classifier's shared-memory limit (its pooled rows: 8 x d fp32, up
+// to d = kCnnMaxFeatures).
+constexpr int kCnnMaxFeatures = 4096;
+cudaError_t cnn_init_attributes();
 
 // ---------------------------------------------------------------- small kernels
 // y [rows, d] bf16 = LayerNorm of x [rows, d] fp32 (eps 1e-6) with statistics

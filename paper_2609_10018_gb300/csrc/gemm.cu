@@ -190,9 +190,12 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int S = args.stages, E = args.cbufs;
   // NB: 1, or 2 when W is held as a bf16 (hi, lo) pair
   const int BSTG = args.b_stage;  // NB planes of bn rows (bn / 2 rows per CTA of a pair)
+  const bool bres = !PAIR && NB == 1 && args.b_resident;
   uint8_t* sA = smem;
-  uint8_t* sB = smem + S * A_STAGE;
-  uint8_t* sC = sB + S * BSTG;  // E staging chunks, or the transpose tiles
+  uint8_t* sB = smem + S * A_STAGE;  // the B ring, or (bres) every k-block of B
+  const int bke = args.k16 ? 16 : BK;  // K values per k-block
+  const int nk = (args.K + bke - 1) / bke;
+  uint8_t* sC = sB + (bres ? nk : S) * BSTG;  // E staging chunks, or the transpose tiles
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + POOL);
   uint64_t* full = bars;
   uint64_t* empty = bars + MAX_STAGES;
@@ -200,12 +203,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   uint64_t* tempty = tfull + 2;
   uint64_t* drain = tempty + 2;
   uint64_t* rfull = drain + 1;  // MAX_CBUFS residual-landed barriers
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(rfull + MAX_CBUFS);
+  uint64_t* bfull = rfull + MAX_CBUFS;  // resident B landed
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bfull + 1);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int M = args.M, N = args.N, bn = args.bn;
-  const int bke = args.k16 ? 16 : BK;  // K values per k-block
-  const int nk = (args.K + bke - 1) / bke;
   constexpr int TM = PAIR ? 2 * BM : BM;  // rows per tile
   const int mt = args.conv ? conv_mtiles(args) : (M + TM - 1) / TM, nt = (N + bn - 1) / bn;
   const int tiles = mt * nt;
@@ -225,6 +227,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     mbar_init(drain, 1);
     for (int e = 0; e < MAX_CBUFS; ++e) mbar_init(&rfull[e], 1);
+    mbar_init(bfull, 1);
     fence_barrier_init();
   }
   if (warp == 0) {
@@ -263,8 +266,13 @@ __global__ void __launch_bounds__(THREADS, 1)
       long issued = 0;
       bool ok = true;
       // pair: the even CTA's full barrier counts both CTAs' bytes
-      const uint32_t bytes =
-          PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2) : (args.conv ? args.cv_a_bytes : A_STAGE) + NB * bn * bke * 2;
+      const uint32_t bytes = PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2)
+                                  : (args.conv ? args.cv_a_bytes : A_STAGE) + (bres ? 0 : NB * bn * bke * 2);
+      const bool b_loaded = bres && t_start < tiles;
+      if (b_loaded) {  // all of W, once: nk k-blocks of the single N tile
+        mbar_expect_tx(bfull, static_cast<uint32_t>(nk) * bn * bke * 2);
+        for (int kb = 0; kb < nk; ++kb) tma_load_2d(sB + kb * BSTG, &tmB, bfull, kb * bke, 0);
+      }
       for (int t = t_start; t < tiles && ok; t += t_stride) {
         const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
         int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
@@ -295,7 +303,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           } else {
             tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
           }
-          tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * bke, n0);
+          if (!bres) tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * bke, n0);
           if constexpr (NB == 2) tma_load_2d(sB + stage * BSTG + BSTG / 2, &tmB2, &full[stage], kb * BK, n0);
           ++issued;
           if (++stage == S) {
@@ -317,6 +325,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         --stage;
         PAIR ? mbar_wait_cluster(&full[stage], phase) : mbar_wait(&full[stage], phase);
       }
+      if (b_loaded) mbar_wait(bfull, 0);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -325,6 +334,8 @@ __global__ void __launch_bounds__(THREADS, 1)
       int stage = 0;
       uint32_t phase = 0;
       bool ok = true, issued = false;
+      // resident B: every tile's MMAs read it; wait for it once
+      if (bres && t_start < tiles && !mbar_wait(bfull, 0)) ok = false;
       int local = 0;
       for (int t = t_start; t < tiles && ok; t += t_stride, ++local) {
         const int acc = local & 1;
@@ -346,7 +357,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a0 = smem_addr(sA + stage * A_STAGE), b0 = smem_addr(sB + stage * BSTG);
+          const uint32_t a0 = smem_addr(sA + stage * A_STAGE), b0 = smem_addr(sB + (bres ? kb : stage) * BSTG);
           if (args.k16) {
             // one K=16 step per k-block: rows of 32 bytes in the 32-byte swizzle,
             // 8-row groups 256 bytes apart
@@ -884,10 +895,22 @@ elasto_status plan_conv_common(GemmPlan* p, const char* who, const void* x, cons
   a.b_planes = 1;
   a.f16 = 1;
   a.pair = 0;
-  a.b_stage = a.bn * BK * 2;
-  a.stages = (POOL - 2 * CBUF) / (A_STAGE + a.b_stage);
-  if (a.stages > MAX_STAGES) a.stages = MAX_STAGES;
-  a.cbufs = (POOL - a.stages * (A_STAGE + a.b_stage)) / CBUF;
+  // one N tile whose whole W fits beside a 4-stage A ring: W is loaded once
+  // per CTA and kept, instead of once per tile and k-block from L2
+  const int nk = taps * cg;
+  const int b_all = nk * a.bn * bke * 2;
+  a.b_resident = (N <= a.bn && 4 * A_STAGE + b_all + 2 * CBUF <= POOL) ? 1 : 0;
+  if (a.b_resident) {
+    a.b_stage = a.bn * bke * 2;  // one k-block of W
+    a.stages = (POOL - 2 * CBUF - b_all) / A_STAGE;
+    if (a.stages > MAX_STAGES) a.stages = MAX_STAGES;
+    a.cbufs = (POOL - a.stages * A_STAGE - b_all) / CBUF;
+  } else {
+    a.b_stage = a.bn * BK * 2;
+    a.stages = (POOL - 2 * CBUF) / (A_STAGE + a.b_stage);
+    if (a.stages > MAX_STAGES) a.stages = MAX_STAGES;
+    a.cbufs = (POOL - a.stages * (A_STAGE + a.b_stage)) / CBUF;
+  }
   if (a.cbufs > MAX_CBUFS) a.cbufs = MAX_CBUFS;
   if (a.cbufs < 2 || rows > BM || a.stages < 2) {
     set_error(std::string(who) + ": shared-memory layout does not fit");
