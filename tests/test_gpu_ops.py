@@ -227,6 +227,11 @@ CONV_CASES = [
     (4, 9, 9, 16, 24, 3, 2, 1, False),       # N below one 64-column chunk, stride 2 (16-channel k-blocks)
     (3, 11, 13, 8, 40, 3, 1, 1, True),       # 8 channels: 16-wide k-blocks, half of each zero
     (2, 20, 20, 16, 64, 4, 1, 2, True),      # 4 x 4 taps on 16 channels (the space-to-depth stem's shape)
+    # stride 1 on 64-channel groups runs as halo tiles (taps = shifted windows of one load per group):
+    (2, 28, 28, 128, 128, 3, 1, 1, True),    # ResNet-50 stage 2 shape: two groups, W streamed per tap
+    (3, 14, 14, 256, 320, 3, 1, 1, False),   # four groups, two N tiles (the second ragged)
+    (2, 9, 30, 72, 64, 5, 1, 2, True),       # 5 x 5, ragged second group, 3 row blocks of 3 rows
+    (2, 10, 12, 64, 64, 3, 1, 0, True),      # no padding
 ]
 
 
