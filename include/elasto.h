@@ -200,7 +200,8 @@ enum {
   ELASTO_Q_WORKSPACE_BYTES = 3,  /* activation workspace for max_batch */
   ELASTO_Q_ARENA_BYTES = 4,      /* total device bytes owned by the handle */
   ELASTO_Q_MODE_MACS = 5,        /* multiply-accumulates per image of the mode */
-  ELASTO_Q_LAUNCHES = 6,         /* kernels one forward of the mode launches */
+  ELASTO_Q_LAUNCHES = 6,         /* kernels one forward of the mode launches (a one-image ViT
+                                    forward adds one per layer: its FC2 runs split-K + a sum) */
   ELASTO_Q_PACKED_TOTAL = 7,     /* device bytes of all modes' packed weights together */
   ELASTO_Q_PREFIX_SHARED = 8     /* 1 if the modes share one prefix-ordered packed copy */
 };

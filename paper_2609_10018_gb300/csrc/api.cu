@@ -407,6 +407,8 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   // k images' worth (k * n >= n + 128 rows) serve every batch
   h->addend_rows = (1 + (128 + n - 1) / n) * n;
   const size_t o_tok = bump.take(size_t(h->addend_rows) * D * 4);
+  // split-K partial sums of the one-image FC2 (kSplitMax x n x D fp32)
+  const size_t o_part = bump.take(size_t(kSplitMax) * n * D * 4);
   const size_t img_bytes = size_t(Bm) * d->img_h * d->img_w * d->img_c * dtype_size(d->weight_dtype);
   const size_t o_img = bump.take(img_bytes), o_logit = bump.take(size_t(Bm) * C * 4);
   const size_t o_status = bump.take(64);
@@ -439,6 +441,7 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   h->head_w = reinterpret_cast<float*>(A + o_head_w);
   h->head_b = reinterpret_cast<float*>(A + o_head_b);
   h->X = reinterpret_cast<float*>(A + o_X);
+  h->splitk_part = reinterpret_cast<float*>(A + o_part);
   h->Y = reinterpret_cast<bf16*>(A + o_Y);
   h->QKV = reinterpret_cast<bf16*>(A + o_QKV);
   h->O = reinterpret_cast<bf16*>(A + o_O);
@@ -836,6 +839,10 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
         vm.launches += 1;
       }
       st = plan_set(lp.fc2, [&](GemmPlan& gp, int rows) {
+        // one image: the 3072-long reduction split over the idle SMs
+        if (rows <= n)
+          return gemm_plan_split_resid(&gp, h->H, Mcap, lp.fc2_w, Dm, lp.f_pad, em.fc2_b[l], h->X, Dm, h->status,
+                                       lp.fc2_w_lo, rows, lp.ld_fc2, h->splitk_part);
         return gemm_plan(&gp, h->H, Mcap, lp.fc2_w, Dm, lp.f_pad, em.fc2_b[l], h->X, Dm, EPI_BIAS_RESID_F32, h->status,
                          lp.fc2_w_lo, rows, lp.ld_fc2);
       });

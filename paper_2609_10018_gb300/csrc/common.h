@@ -121,6 +121,9 @@ struct GemmArgs {
                                              // operands in the 32-byte swizzle
   int b_resident;                            // 1: all of W (one N tile) is loaded once per CTA and kept in
                                              // shared memory; the ring carries A only
+  int ksplit;                                // > 1: split-K, tile t reduces k-block range t / (mt * nt) of
+                                             // ksplit and writes its fp32 partial to out + split * split_stride
+  long long split_stride;                    // elements between the partial sums of two splits
 };
 
 struct GemmPlan {
@@ -130,6 +133,11 @@ struct GemmPlan {
   GemmArgs args;          // M here is the capacity the A map was encoded for
   int epi = 0;
   bool valid = false;
+  // split-K residual plan (gemm_plan_split_resid): after the kernel,
+  // rout[r, c] += rbias[c] + sum over splits of the partials, in split order
+  const float* rbias = nullptr;
+  float* rout = nullptr;
+  int rldo = 0, rcap = 0;  // rout row stride; rows the partial buffer holds
 };
 
 // Pick the N tile for an M x N problem.
@@ -145,7 +153,18 @@ int gemm_pick_bn(int M, int N, int step = 32, bool pair = false);
 // first K columns of a wider matrix (a mode's prefix of a shared packed copy).
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
                         void* out, int ldo, int epi, int* status, const bf16* W_lo = nullptr, int M_hint = 0,
-                        int ldw = 0);
+                        int ldw = 0, int bn_force = 0);
+// EPI_BIAS_RESID_F32 (out[r, :] += A W^T + bias) for at most M_rows rows with
+// the reduction split over up to kSplitMax CTAs per tile when the tiles alone
+// would leave most SMs idle (a long K on a few rows: FC2 at batch 1). The
+// partial sums go to part [ksplit, M_rows, N] fp32 (kSplitMax * M_rows * N
+// floats), then a second launch adds them in split order with the bias to
+// out: deterministic. Falls back to the single-pass plan when splitting
+// would not spread the work.
+constexpr int kSplitMax = 8;
+elasto_status gemm_plan_split_resid(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K,
+                                    const float* bias, float* out, int ldo, int* status, const bf16* W_lo, int M_rows,
+                                    int ldw, float* part);
 
 // Launch plans of one GEMM for a few batch sizes: the forward picks the plan
 // made for the smallest row count that covers its rows.

@@ -28,6 +28,8 @@
 //      embedding) transpose through padded shared memory for row-contiguous
 //      stores.
 //  Every mbarrier wait is bounded; a timeout records ELASTO_ERR_TIMEOUT.
+#include <algorithm>
+
 #include "common.h"
 #include "ptx.cuh"
 
@@ -210,7 +212,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int M = args.M, N = args.N, bn = args.bn;
   constexpr int TM = PAIR ? 2 * BM : BM;  // rows per tile
   const int mt = args.conv ? conv_mtiles(args) : (M + TM - 1) / TM, nt = (N + bn - 1) / bn;
-  const int tiles = mt * nt;
+  // split-K: tile t covers output tile t % (mt * nt) and k-block range
+  // t / (mt * nt) of ks (ks = 1: the whole reduction)
+  const int ks = args.ksplit > 1 ? args.ksplit : 1;
+  const int mn_tiles = mt * nt;
+  const int tiles = mn_tiles * ks;
   const int rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;  // this CTA's row half of a pair tile
   const int t_start = PAIR ? static_cast<int>(cluster_id_x()) : static_cast<int>(blockIdx.x);
   const int t_stride = PAIR ? static_cast<int>(cluster_count_x()) : static_cast<int>(gridDim.x);
@@ -274,10 +280,11 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int kb = 0; kb < nk; ++kb) tma_load_2d(sB + kb * BSTG, &tmB, bfull, kb * bke, 0);
       }
       for (int t = t_start; t < tiles && ok; t += t_stride) {
-        const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
+        const int tq = t % mn_tiles, sp = t / mn_tiles;
+        const int m0 = m_tile(args, tq / nt, mt) * TM + rank * BM, n0 = (tq % nt) * bn;
         int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
-        if (args.conv) conv_tile(args, m_tile(args, t / nt, mt), cb0, cy0, cx0);
-        for (int kb = 0; kb < nk; ++kb) {
+        if (args.conv) conv_tile(args, m_tile(args, tq / nt, mt), cb0, cy0, cx0);
+        for (int kb = sp * nk / ks; kb < (sp + 1) * nk / ks; ++kb) {
           if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
             ok = false;
             break;
@@ -351,7 +358,8 @@ __global__ void __launch_bounds__(THREADS, 1)
           if constexpr (PAIR) mbar_arrive_cluster(cluster_map(smem_addr(&tfull[acc]), 1));
           continue;
         }
-        for (int kb = 0; kb < nk; ++kb) {
+        const int kb0 = (t / mn_tiles) * nk / ks, kb1 = (t / mn_tiles + 1) * nk / ks;
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!(PAIR ? mbar_wait_cluster(&full[stage], phase) : mbar_wait(&full[stage], phase))) {
             ok = false;
             break;
@@ -362,16 +370,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             // one K=16 step per k-block: rows of 32 bytes in the 32-byte swizzle,
             // 8-row groups 256 bytes apart
             if constexpr (!PAIR && NB == 1)
-              tc_mma(dtm, sdesc_sw32(a0, 16, 256), sdesc_sw32(b0, 16, 256), idesc, kb != 0);
+              tc_mma(dtm, sdesc_sw32(a0, 16, 256), sdesc_sw32(b0, 16, 256), idesc, kb != kb0);
           } else
 #pragma unroll
           for (int k = 0; k < BK / 16; ++k) {
             if constexpr (PAIR) {
               tc_mma_pair(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
-                          (kb | k) != 0);
+                          kb != kb0 || k != 0);
             } else {
               tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
-                     (kb | k) != 0);
+                     kb != kb0 || k != 0);
               if constexpr (NB == 2)  // low half of the weights: acc += A . W_lo^T
                 tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + BSTG / 2 + k * 32, 16, 1024),
                        idesc, 1u);
@@ -600,7 +608,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         break;
       }
       tc_fence_after();
-      const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
+      const int tq = t % mn_tiles;
+      const int m0 = m_tile(args, tq / nt, mt) * TM + rank * BM, n0 = (tq % nt) * bn;
       const int row0 = m0 + q * 32;
       for (int c = 0; c < bn; c += 32) {
         if (n0 + c >= N) break;
@@ -619,7 +628,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           const int col = n0 + c + lane;
           const bool cok = col < N;
           const float bv = (cok && args.bias) ? args.bias[col] : 0.0f;
-          float* out = static_cast<float*>(args.out);
+          float* out = static_cast<float*>(args.out) + (t / mn_tiles) * args.split_stride;
           if constexpr (EPI == EPI_BIAS_F32) {
 #pragma unroll 8
             for (int i = 0; i < 32; ++i) {
@@ -659,6 +668,38 @@ __global__ void __launch_bounds__(THREADS, 1)
   }
 }
 
+// Split-K residual: out[r, c] += (sum over splits of part[s][r, c]) + bias[c],
+// the splits added in order, the sum and bias associated as in the one-pass
+// RESID_F32 epilogue (x + (acc + b)). One thread per 4 columns of a row.
+__global__ void splitk_reduce_kernel(const float* __restrict__ part, int ks, long long stride, int M, int N,
+                                     const float* __restrict__ bias, float* __restrict__ out, int ldo) {
+  pdl_wait();
+  pdl_trigger();
+  const int n4 = N / 4;
+  const size_t total = static_cast<size_t>(M) * n4;
+  for (size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+       i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const size_t r = i / n4;
+    const int c = static_cast<int>(i - r * n4) * 4;
+    float4 acc = *reinterpret_cast<const float4*>(part + r * N + c);
+    for (int sp = 1; sp < ks; ++sp) {
+      const float4 v = *reinterpret_cast<const float4*>(part + sp * stride + r * N + c);
+      acc.x += v.x;
+      acc.y += v.y;
+      acc.z += v.z;
+      acc.w += v.w;
+    }
+    const float4 b = bias ? *reinterpret_cast<const float4*>(bias + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+    float4* o = reinterpret_cast<float4*>(out + r * ldo + c);
+    float4 x = *o;
+    x.x += acc.x + b.x;
+    x.y += acc.y + b.y;
+    x.z += acc.z + b.z;
+    x.w += acc.w + b.w;
+    *o = x;
+  }
+}
+
 template <int EPI, int NB, bool PAIR>
 cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   GemmArgs a = p.args;
@@ -695,7 +736,7 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
     cfg.numAttrs = 2;
     return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<EPI, NB, true>, p.tmA, p.tmB, p.tmB2, p.tmC, p.tmR, a);
   } else {
-    const int tiles = (a.conv ? conv_mtiles(a) : (M + BM - 1) / BM) * nt;
+    const int tiles = (a.conv ? conv_mtiles(a) : (M + BM - 1) / BM) * nt * (a.ksplit > 1 ? a.ksplit : 1);
     const int grid = tiles < num_sms() ? tiles : num_sms();
     return launch_pdl(gemm_tc_kernel<EPI, NB, false>, dim3(grid), dim3(THREADS), SMEM_BYTES, s, p.tmA, p.tmB, p.tmB2,
                       p.tmC, p.tmR, a);
@@ -756,7 +797,8 @@ int gemm_pick_bn(int M, int N, int step, bool pair) {
 }
 
 elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K, const float* bias,
-                        void* out, int ldo, int epi, int* status, const bf16* W_lo, int M_hint, int ldw) {
+                        void* out, int ldo, int epi, int* status, const bf16* W_lo, int M_hint, int ldw,
+                        int bn_force) {
   if (!p || M_cap <= 0 || N <= 0 || K < 0 || !out || (K > 0 && (!A || !W))) {
     set_error("gemm_plan: invalid arguments");
     return ELASTO_ERR_INVALID_ARG;
@@ -785,7 +827,7 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
   const bool pair = tma_out && !W_lo && Mt >= 2 * BM && K >= 1536;
   a.pair = pair ? 1 : 0;
   // bf16 staging chunks are 64 columns wide: their tiles are multiples of 64
-  a.bn = gemm_pick_bn(Mt, N, (tma_out && !f32_out) ? 64 : 32, pair);
+  a.bn = bn_force > 0 ? bn_force : gemm_pick_bn(Mt, N, (tma_out && !f32_out) ? 64 : 32, pair);
   // one B stage holds exactly the tile's rows (both planes); the freed bytes
   // become a deeper operand ring for narrow tiles
   a.b_stage = pair ? (a.bn / 2) * BK * 2 : (W_lo ? 2 : 1) * a.bn * BK * 2;
@@ -838,6 +880,40 @@ elasto_status gemm_plan(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, in
     }
   }
   p->valid = true;
+  return ELASTO_OK;
+}
+
+elasto_status gemm_plan_split_resid(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K,
+                                    const float* bias, float* out, int ldo, int* status, const bf16* W_lo, int M_rows,
+                                    int ldw, float* part) {
+  const int sms = num_sms() > 0 ? num_sms() : 148;
+  const int rows = (M_rows > 0 && M_rows < M_cap) ? M_rows : M_cap;
+  const int mt = (rows + BM - 1) / BM, nk = (K + BK - 1) / BK;
+  // the N tile and split count with the fewest k-blocks per CTA, every
+  // split keeping at least 4 k-blocks
+  int best_bn = 0, best_ks = 1, best_kb = nk + 1;
+  for (int bn : {64, 32}) {
+    const int tiles = mt * ((N + bn - 1) / bn);
+    const int ks = std::min({kSplitMax, sms / std::max(tiles, 1), nk / 4});
+    if (ks < 2) continue;
+    const int kb = (nk + ks - 1) / ks;
+    if (kb < best_kb) {
+      best_kb = kb;
+      best_bn = bn;
+      best_ks = ks;
+    }
+  }
+  if (best_bn == 0 || !part || N % 4 != 0 || ldo % 4 != 0)
+    return gemm_plan(p, A, M_cap, W, N, K, bias, out, ldo, EPI_BIAS_RESID_F32, status, W_lo, M_rows, ldw);
+  elasto_status st =
+      gemm_plan(p, A, M_cap, W, N, K, nullptr, part, N, EPI_BIAS_F32, status, W_lo, rows, ldw, best_bn);
+  if (st != ELASTO_OK) return st;
+  p->args.ksplit = best_ks;
+  p->args.split_stride = static_cast<long long>(rows) * N;
+  p->rbias = bias;
+  p->rout = out;
+  p->rldo = ldo;
+  p->rcap = rows;
   return ELASTO_OK;
 }
 
@@ -1016,8 +1092,9 @@ elasto_status gemm_set_residual_source(GemmPlan* p, const void* src, int M_cap, 
   return ELASTO_OK;
 }
 
-cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s) {
-  if (M <= 0) return cudaSuccess;
+namespace {
+
+cudaError_t gemm_launch_main(const GemmPlan& p, int M, cudaStream_t s) {
   const bool two = p.args.b_planes == 2, pair = p.args.pair != 0;
 #define CASE(E) \
   case E: return two ? launch_epi<E, 2, false>(p, M, s) : launch_epi<E, 1, false>(p, M, s);
@@ -1040,6 +1117,20 @@ cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s) {
 #undef CASE_PAIR
     default: return cudaErrorInvalidValue;
   }
+}
+
+}  // namespace
+
+cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s) {
+  if (M <= 0) return cudaSuccess;
+  if (p.args.ksplit <= 1) return gemm_launch_main(p, M, s);
+  if (M > p.rcap) return cudaErrorInvalidValue;  // the partial buffer holds rcap rows
+  cudaError_t e = gemm_launch_main(p, M, s);
+  if (e != cudaSuccess) return e;
+  const size_t work = static_cast<size_t>(M) * (p.args.N / 4);
+  const unsigned grid = static_cast<unsigned>(std::min<size_t>((work + 255) / 256, 4096));
+  return launch_pdl(splitk_reduce_kernel, dim3(grid), dim3(256), 0, s, static_cast<const float*>(p.args.out),
+                    p.args.ksplit, p.args.split_stride, M, p.args.N, p.rbias, p.rout, p.rldo);
 }
 
 }  // namespace elasto

@@ -67,6 +67,7 @@ struct elasto_s {
   std::vector<float*> ln1_w, ln1_b, proj_b, ln2_w, ln2_b, fc2_b;
   // workspace
   float* X = nullptr;
+  float* splitk_part = nullptr;  // split-K partial sums of the one-image FC2
   elasto::bf16 *Y = nullptr, *QKV = nullptr, *O = nullptr, *H = nullptr, *P = nullptr;
   // Per-token addend of the patch projection (cls + pos[0] on class tokens,
   // pos[t] + b_pe on patch tokens) for k = 1 + ceil(128 / n) images: it is

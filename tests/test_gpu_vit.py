@@ -106,6 +106,33 @@ def test_vit_b_small_batches(batch):
     _sampled_parity(synth.VIT_B, batch, np.array([0, batch - 1]), modes=[0, 4])
 
 
+def test_one_image_on_larger_handles_all_modes(tiny):
+    """A one-image forward on handles built for more images takes the
+    one-image plans (FC2's reduction split over idle SMs, the partial sums
+    added in a second launch): every mode against the oracle, and within the
+    same bound of that image's logits inside a larger batch (the split sums
+    FC2 in another order, and a last-bit change of the fp32 residual can move
+    a later bf16 rounding)."""
+    for cfg, w, wide, tables, big in [(*tiny, 8), _vit_s_setup() + (64,)]:
+        img = synth.make_images(cfg, big)
+        with binding.ElasticModel.vit(cfg, w, tables, max_batch=big) as model:
+            x1, xb = dev(img[:1]), dev(img)
+            for m, t in enumerate(tables):
+                one = _run(model, x1, 1, cfg.classes, m)
+                ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img[:1])
+                assert rel_err(one, ref) <= TOL, (cfg.name, m)
+                many = _run(model, xb, big, cfg.classes, m)[:1]
+                assert rel_err(one, many) <= TOL, (cfg.name, m)
+                # repeatable bit for bit (the split sums in a fixed order)
+                assert np.array_equal(_run(model, x1, 1, cfg.classes, m), one)
+
+
+def _vit_s_setup():
+    cfg = synth.VIT_S
+    w = synth.make_vit_weights(cfg)
+    return cfg, w, ov.widen_all(w), synth.make_vit_tables(cfg)
+
+
 def test_mode_switch_between_enqueued_forwards(tiny):
     """set_mode only affects forwards enqueued after it; no sync in between."""
     import torch
