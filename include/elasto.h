@@ -201,7 +201,9 @@ enum {
   ELASTO_Q_ARENA_BYTES = 4,      /* total device bytes owned by the handle */
   ELASTO_Q_MODE_MACS = 5,        /* multiply-accumulates per image of the mode */
   ELASTO_Q_LAUNCHES = 6,         /* kernels one forward of the mode launches (a one-image ViT
-                                    forward adds one per layer: its FC2 runs split-K + a sum) */
+                                    forward launches at most one more: its out-projection and FC2 run
+                                    split-K, their partial-sum launches compute the LayerNorms
+                                    that follow, and the last FC2's sum stands alone) */
   ELASTO_Q_PACKED_TOTAL = 7,     /* device bytes of all modes' packed weights together */
   ELASTO_Q_PREFIX_SHARED = 8     /* 1 if the modes share one prefix-ordered packed copy */
 };

@@ -826,6 +826,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
         vm.launches += 2;
       }
       st = plan_set(lp.proj, [&](GemmPlan& gp, int rows) {
+        // one image: the reduction split over idle SMs, and LN2 computed by
+        // the launch that adds the partial sums
+        if (rows <= n) {
+          const elasto_status r = gemm_plan_split_resid(&gp, h->O, Mcap, lp.proj_w, Dm, lp.w, em.proj_b[l], h->X, Dm,
+                                                        h->status, lp.proj_w_lo, rows, lp.ld_proj, h->splitk_part);
+          if (r == ELASTO_OK) gemm_split_fuse_layernorm(&gp, em.ln2_w[l], em.ln2_b[l], h->Y, em.d);
+          return r;
+        }
         return gemm_plan(&gp, h->O, Mcap, lp.proj_w, Dm, lp.w, em.proj_b[l], h->X, Dm, EPI_BIAS_RESID_F32, h->status,
                          lp.proj_w_lo, rows, lp.ld_proj);
       });
@@ -839,10 +847,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
         vm.launches += 1;
       }
       st = plan_set(lp.fc2, [&](GemmPlan& gp, int rows) {
-        // one image: the 3072-long reduction split over the idle SMs
-        if (rows <= n)
-          return gemm_plan_split_resid(&gp, h->H, Mcap, lp.fc2_w, Dm, lp.f_pad, em.fc2_b[l], h->X, Dm, h->status,
-                                       lp.fc2_w_lo, rows, lp.ld_fc2, h->splitk_part);
+        // one image: the 3072-long reduction split over the idle SMs, and
+        // the next layer's LN1 computed by the launch that adds the partials
+        if (rows <= n) {
+          const elasto_status r = gemm_plan_split_resid(&gp, h->H, Mcap, lp.fc2_w, Dm, lp.f_pad, em.fc2_b[l], h->X,
+                                                        Dm, h->status, lp.fc2_w_lo, rows, lp.ld_fc2, h->splitk_part);
+          if (r == ELASTO_OK && l + 1 < L) gemm_split_fuse_layernorm(&gp, em.ln1_w[l + 1], em.ln1_b[l + 1], h->Y, em.d);
+          return r;
+        }
         return gemm_plan(&gp, h->H, Mcap, lp.fc2_w, Dm, lp.f_pad, em.fc2_b[l], h->X, Dm, EPI_BIAS_RESID_F32, h->status,
                          lp.fc2_w_lo, rows, lp.ld_fc2);
       });
@@ -897,8 +909,10 @@ elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int b
   const double ln_bytes = double(M) * Dm * (4 + 2);
   for (int l = 0; l < d.layers; ++l) {
     const VitLayerPack& lp = vm.layers[l];
-    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, Dm, 0, 0, ln_bytes),
-                  layernorm_launch(h->X, em.ln1_w[l], em.ln1_b[l], h->Y, M, Dm, em.d, s));
+    // LN1 / LN2 are skipped where the previous GEMM's split-K sum computed them
+    if (l == 0 || !vm.layers[l - 1].fc2.pick(M).ln_y)
+      ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, Dm, 0, 0, ln_bytes),
+                    layernorm_launch(h->X, em.ln1_w[l], em.ln1_b[l], h->Y, M, Dm, em.d, s));
     if (lp.w > 0) {
       ELASTO_LAUNCH(gemm_rec(l, M, 3 * lp.w, Dm, 2, false), gemm_launch(lp.qkv.pick(M), M, s));
       ELASTO_LAUNCH(make_rec(ELASTO_K_ATTENTION, l, M, lp.w, n, 2.0 * batch * n * n * lp.w,
@@ -906,8 +920,9 @@ elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int b
                     attn_launch(lp.attn, batch, s));
     }
     ELASTO_LAUNCH(gemm_rec(l, M, Dm, lp.w, 4, true), gemm_launch(lp.proj.pick(M), M, s));
-    ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, Dm, 0, 0, ln_bytes),
-                  layernorm_launch(h->X, em.ln2_w[l], em.ln2_b[l], h->Y, M, Dm, em.d, s));
+    if (!lp.proj.pick(M).ln_y)
+      ELASTO_LAUNCH(make_rec(ELASTO_K_LAYERNORM, l, M, Dm, 0, 0, ln_bytes),
+                    layernorm_launch(h->X, em.ln2_w[l], em.ln2_b[l], h->Y, M, Dm, em.d, s));
     if (lp.f > 0) ELASTO_LAUNCH(gemm_rec(l, M, lp.f_pad, Dm, 2, false), gemm_launch(lp.fc1.pick(M), M, s));
     ELASTO_LAUNCH(gemm_rec(l, M, Dm, lp.f_pad, 4, true), gemm_launch(lp.fc2.pick(M), M, s));
   }

@@ -138,6 +138,12 @@ struct GemmPlan {
   const float* rbias = nullptr;
   float* rout = nullptr;
   int rldo = 0, rcap = 0;  // rout row stride; rows the partial buffer holds
+  // optional LayerNorm of the finished rows, fused into that sum
+  // (gemm_split_fuse_layernorm): ln_y = LN(rout) over the first ln_d channels
+  const float* ln_g = nullptr;
+  const float* ln_b = nullptr;
+  bf16* ln_y = nullptr;
+  int ln_d = 0;
 };
 
 // Pick the N tile for an M x N problem.
@@ -165,6 +171,13 @@ constexpr int kSplitMax = 8;
 elasto_status gemm_plan_split_resid(GemmPlan* p, const bf16* A, int M_cap, const bf16* W, int N, int K,
                                     const float* bias, float* out, int ldo, int* status, const bf16* W_lo, int M_rows,
                                     int ldw, float* part);
+// For a split plan (does nothing otherwise, and says so by returning false):
+// the launch that adds the partial sums also writes y = LayerNorm(out row)
+// (gamma g, beta b, statistics over the first d_true of the N channels, the
+// rest zero padding), the LayerNorm layernorm_launch computes (summed in
+// another order), so the caller skips that launch. Needs ldo == N,
+// N % 64 == 0, N <= 1024.
+bool gemm_split_fuse_layernorm(GemmPlan* p, const float* g, const float* b, bf16* y, int d_true);
 
 // Launch plans of one GEMM for a few batch sizes: the forward picks the plan
 // made for the smallest row count that covers its rows.

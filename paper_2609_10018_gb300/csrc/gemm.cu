@@ -700,6 +700,62 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int ks, lon
   }
 }
 
+// Sum over the threads of a block of nw warps (nw <= 32); red: nw floats of
+// shared memory. Every thread gets the total.
+__device__ __forceinline__ float block_sum(float v, float* red, int nw) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = lane < nw ? red[lane] : 0.0f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+  __syncthreads();  // red is reused by the next call
+  return t;
+}
+
+// The same sum, and then the LayerNorm of each finished row: one block of
+// N / 2 threads per row, two channels per thread (all the row's partial sums
+// in flight at once). Statistics as layernorm_kernel takes them (mean over
+// the first d_true channels, centred sum of squares less the zero padding's
+// pad * mean^2, eps 1e-6), summed in another order.
+__global__ void __launch_bounds__(512) splitk_reduce_ln_kernel(const float* __restrict__ part, int ks,
+                                                               long long stride, int N,
+                                                               const float* __restrict__ bias,
+                                                               float* __restrict__ out, const float* __restrict__ g,
+                                                               const float* __restrict__ b, bf16* __restrict__ y,
+                                                               float inv_d, float pad) {
+  __shared__ float red[32];
+  pdl_wait();
+  pdl_trigger();
+  const size_t e = static_cast<size_t>(blockIdx.x) * N + 2 * threadIdx.x;
+  float2 p2[kSplitMax];
+#pragma unroll
+  for (int sp = 0; sp < kSplitMax; ++sp)
+    p2[sp] = sp < ks ? *reinterpret_cast<const float2*>(part + sp * stride + e) : make_float2(0.f, 0.f);
+  float2 acc = p2[0];
+#pragma unroll
+  for (int sp = 1; sp < kSplitMax; ++sp)
+    if (sp < ks) {
+      acc.x += p2[sp].x;
+      acc.y += p2[sp].y;
+    }
+  const float2 bb = bias ? reinterpret_cast<const float2*>(bias)[threadIdx.x] : make_float2(0.f, 0.f);
+  float2* o = reinterpret_cast<float2*>(out + e);
+  float2 x = *o;
+  x.x += acc.x + bb.x;
+  x.y += acc.y + bb.y;
+  *o = x;
+  const int nw = blockDim.x >> 5;
+  const float mean = block_sum(x.x + x.y, red, nw) * inv_d;
+  const float a = x.x - mean, c = x.y - mean;
+  const float rstd = rsqrtf((block_sum(a * a + c * c, red, nw) - pad * mean * mean) * inv_d + 1e-6f);
+  const float2 gg = reinterpret_cast<const float2*>(g)[threadIdx.x];
+  const float2 be = reinterpret_cast<const float2*>(b)[threadIdx.x];
+  reinterpret_cast<uint32_t*>(y)[e / 2] = pack_bf16x2(a * rstd * gg.x + be.x, c * rstd * gg.y + be.y);
+}
+
 template <int EPI, int NB, bool PAIR>
 cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   GemmArgs a = p.args;
@@ -917,6 +973,17 @@ elasto_status gemm_plan_split_resid(GemmPlan* p, const bf16* A, int M_cap, const
   return ELASTO_OK;
 }
 
+bool gemm_split_fuse_layernorm(GemmPlan* p, const float* g, const float* b, bf16* y, int d_true) {
+  if (!p || p->args.ksplit <= 1 || !g || !b || !y || p->rldo != p->args.N || p->args.N % 64 != 0 ||
+      p->args.N > 1024 || d_true <= 0 || d_true > p->args.N)
+    return false;
+  p->ln_g = g;
+  p->ln_b = b;
+  p->ln_y = y;
+  p->ln_d = d_true;
+  return true;
+}
+
 namespace {
 
 // The part both convolution plans share. A is read through the 4D map
@@ -1127,6 +1194,12 @@ cudaError_t gemm_launch(const GemmPlan& p, int M, cudaStream_t s) {
   if (M > p.rcap) return cudaErrorInvalidValue;  // the partial buffer holds rcap rows
   cudaError_t e = gemm_launch_main(p, M, s);
   if (e != cudaSuccess) return e;
+  if (p.ln_y) {
+    const float inv_d = 1.0f / static_cast<float>(p.ln_d), pad = static_cast<float>(p.args.N - p.ln_d);
+    return launch_pdl(splitk_reduce_ln_kernel, dim3(M), dim3(p.args.N / 2), 0, s,
+                      static_cast<const float*>(p.args.out), p.args.ksplit, p.args.split_stride, p.args.N, p.rbias,
+                      p.rout, p.ln_g, p.ln_b, p.ln_y, inv_d, pad);
+  }
   const size_t work = static_cast<size_t>(M) * (p.args.N / 4);
   const unsigned grid = static_cast<unsigned>(std::min<size_t>((work + 255) / 256, 4096));
   return launch_pdl(splitk_reduce_kernel, dim3(grid), dim3(256), 0, s, static_cast<const float*>(p.args.out),

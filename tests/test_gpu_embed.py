@@ -94,6 +94,24 @@ def test_vit_b_embedding_pruned_mode_sampled():
         assert err <= TOL
 
 
+def test_one_image_embedding_pruned_modes():
+    """One image on a larger handle (split-K out-projection and FC2 whose
+    partial-sum launches also compute the LayerNorms over the kept channels)
+    for pruned widths that are and are not multiples of 64."""
+    cfg = synth.VIT_S
+    w = synth.make_vit_weights(cfg)
+    wide = ov.widen_all(w)
+    tables = synth.with_embedding(cfg, synth.make_vit_tables(cfg), [None, 320, 200, 96])
+    img = synth.make_images(cfg, 2, seed=8)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=16) as model:
+        for i in range(2):
+            x = dev(img[i:i + 1])
+            for m, t in enumerate(tables):
+                err = rel_err(_run(model, x, 1, cfg.classes, m), _ref(wide, cfg, t, img[i:i + 1]))
+                print(f"vit_s one image {i} mode {m}: err {err:.2e}")
+                assert err <= TOL
+
+
 def test_embedding_pruned_packed_layouts_exact():
     """Packed buffers of a pruned mode are the stored weights' kept rows and
     columns, bit for bit (bf16-stored ViT-S)."""
