@@ -212,9 +212,11 @@ __global__ void __launch_bounds__(THREADS, 1)
   const int M = args.M, N = args.N, bn = args.bn;
   constexpr int TM = PAIR ? 2 * BM : BM;  // rows per tile
   const int mt = args.conv ? conv_mtiles(args) : (M + TM - 1) / TM, nt = (N + bn - 1) / bn;
-  // split-K: tile t covers output tile t % (mt * nt) and k-block range
-  // t / (mt * nt) of ks (ks = 1: the whole reduction)
-  const int ks = args.ksplit > 1 ? args.ksplit : 1;
+  // split-K (fp32 partial outputs only): tile t covers output tile
+  // t % (mt * nt) and k-block range t / (mt * nt) of ks. Every other
+  // epilogue has ks = 1 at compile time and no division on its tile path.
+  constexpr bool kSplit = EPI == EPI_BIAS_F32;
+  const int ks = kSplit && args.ksplit > 1 ? args.ksplit : 1;
   const int mn_tiles = mt * nt;
   const int tiles = mn_tiles * ks;
   const int rank = PAIR ? static_cast<int>(cluster_ctarank()) : 0;  // this CTA's row half of a pair tile
@@ -280,11 +282,12 @@ __global__ void __launch_bounds__(THREADS, 1)
         for (int kb = 0; kb < nk; ++kb) tma_load_2d(sB + kb * BSTG, &tmB, bfull, kb * bke, 0);
       }
       for (int t = t_start; t < tiles && ok; t += t_stride) {
-        const int tq = t % mn_tiles, sp = t / mn_tiles;
+        const int tq = kSplit ? t % mn_tiles : t;
+        const int kb0 = kSplit ? (t / mn_tiles) * nk / ks : 0, kb1 = kSplit ? (t / mn_tiles + 1) * nk / ks : nk;
         const int m0 = m_tile(args, tq / nt, mt) * TM + rank * BM, n0 = (tq % nt) * bn;
         int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
         if (args.conv) conv_tile(args, m_tile(args, tq / nt, mt), cb0, cy0, cx0);
-        for (int kb = sp * nk / ks; kb < (sp + 1) * nk / ks; ++kb) {
+        for (int kb = kb0; kb < kb1; ++kb) {
           if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
             ok = false;
             break;
@@ -358,7 +361,7 @@ __global__ void __launch_bounds__(THREADS, 1)
           if constexpr (PAIR) mbar_arrive_cluster(cluster_map(smem_addr(&tfull[acc]), 1));
           continue;
         }
-        const int kb0 = (t / mn_tiles) * nk / ks, kb1 = (t / mn_tiles + 1) * nk / ks;
+        const int kb0 = kSplit ? (t / mn_tiles) * nk / ks : 0, kb1 = kSplit ? (t / mn_tiles + 1) * nk / ks : nk;
         for (int kb = kb0; kb < kb1; ++kb) {
           if (!(PAIR ? mbar_wait_cluster(&full[stage], phase) : mbar_wait(&full[stage], phase))) {
             ok = false;
