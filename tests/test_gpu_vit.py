@@ -125,6 +125,10 @@ def test_one_image_on_larger_handles_all_modes(tiny):
                 assert rel_err(one, many) <= TOL, (cfg.name, m)
                 # repeatable bit for bit (the split sums in a fixed order)
                 assert np.array_equal(_run(model, x1, 1, cfg.classes, m), one)
+                # eight images: the 8-image plans split the residual GEMMs too
+                eight = _run(model, dev(img[:8]), 8, cfg.classes, m)
+                ref8 = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img[[0, 7]])
+                assert rel_err(eight[[0, 7]], ref8) <= TOL, (cfg.name, m)
 
 
 def _vit_s_setup():
