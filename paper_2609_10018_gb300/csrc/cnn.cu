@@ -233,26 +233,39 @@ __global__ void maxpool_kernel(const uint4* __restrict__ src, int H, int W, int 
 }
 
 // Global average pool: dst[b, c] = mean over the HW pixels of src[b, :, c]
-// (f16 in, fp32 sums and result). Item t = b * C8 + c8.
+// (f16 in, fp32 sums and result). Item t = b * C8 + c8 (8 channels) is
+// taken by the 4 adjacent threads 4t .. 4t + 3: thread j sums the pixels
+// p = j (mod 4), the four partial sums are combined with shuffles inside
+// the 4-lane group, and thread j writes channels 2j, 2j + 1.
 __global__ void avgpool_kernel(const uint4* __restrict__ src, int HW, int C8, size_t total, float* __restrict__ dst) {
   pdl_wait();
   pdl_trigger();
-  for (size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < total;
-       t += static_cast<size_t>(gridDim.x) * blockDim.x) {
+  const unsigned group = 0xFu << (threadIdx.x & 28);  // this thread's 4-lane group
+  for (size_t u = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; u < 4 * total;
+       u += static_cast<size_t>(gridDim.x) * blockDim.x) {
+    const size_t t = u >> 2;
+    const int j = static_cast<int>(u & 3);
     const int c8 = static_cast<int>(t % C8);
     const size_t b = t / C8;
     float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-#pragma unroll 7
-    for (int p = 0; p < HW; ++p) {
+#pragma unroll 4
+    for (int p = j; p < HW; p += 4) {
       float f[8];
       unpack8(src[(b * HW + p) * C8 + c8], f);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) s[j] += f[j];
+      for (int k = 0; k < 8; ++k) s[k] += f[k];
+    }
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      s[k] += __shfl_xor_sync(group, s[k], 1);
+      s[k] += __shfl_xor_sync(group, s[k], 2);
     }
     const float inv = 1.0f / static_cast<float>(HW);
-    float4* o = reinterpret_cast<float4*>(dst + t * 8);
-    o[0] = make_float4(s[0] * inv, s[1] * inv, s[2] * inv, s[3] * inv);
-    o[1] = make_float4(s[4] * inv, s[5] * inv, s[6] * inv, s[7] * inv);
+    float2 w = make_float2(s[0], s[1]);
+#pragma unroll
+    for (int k = 1; k < 4; ++k)
+      if (k == j) w = make_float2(s[2 * k], s[2 * k + 1]);
+    reinterpret_cast<float2*>(dst + t * 8)[j] = make_float2(w.x * inv, w.y * inv);
   }
 }
 
@@ -794,7 +807,7 @@ elasto_status cnn_forward(CnnModel* m, int mode, cudaStream_t s, const void* ima
   {
     const size_t total = size_t(B) * (cfin / 8);
     CNN_LAUNCH(rec(ELASTO_K_POOL, nblk, B, cfin, 0, 0, double(B) * hw * cfin * 2 + double(B) * cfin * 4),
-               launch_pdl(avgpool_kernel, dim3(grid_for(total)), dim3(256), 0, s, reinterpret_cast<const uint4*>(xfin),
+               launch_pdl(avgpool_kernel, dim3(grid_for(4 * total)), dim3(256), 0, s, reinterpret_cast<const uint4*>(xfin),
                           hw, cfin / 8, total, m->pooled));
   }
   {
