@@ -7,26 +7,35 @@
 // just the problem's N or K.
 //
 // Design (sm_103a):
-//  - persistent grid, one CTA per SM, static round-robin over 128 x bn tiles
-//    (N tile index fastest so the CTAs running together share A rows in L2);
-//  - warp 0 lane 0: TMA producer, ring of 128x64 (A) and bn x 64 (B) bf16
-//    tiles with the 128-byte swizzle, one mbarrier pair per stage;
+//  - persistent grid, one CTA per SM (or one CTA pair per two SMs), static
+//    round-robin over 128 x bn tiles (N tile index fastest so the CTAs
+//    running together share A rows in L2; m_reverse runs the rows backwards);
+//  - warp 0 lane 0: TMA producer, ring of 128x64 (A) and bn x 64 (B) bf16 or
+//    f16 tiles with the 128-byte swizzle, one mbarrier pair per stage. W may
+//    instead be loaded once per CTA and kept (b_resident: one N tile);
 //  - warp 1 lane 0: issues tcgen05.mma (M=128, N=bn, K=16) into one of two
 //    TMEM accumulators (2 x 256 fp32 columns), commits stages back to the
-//    producer and finished accumulators to the epilogue;
-//  - warps 2-5: epilogue. Each warp owns one 32-lane quarter of TMEM (= 32
-//    rows of the tile); each thread owns one row.
+//    producer and finished accumulators to the epilogue. K >= 1536 on
+//    256-row tiles: CTA pairs (cta_group::2, M = 256, each CTA holds half of
+//    B);
+//  - warps 2-17: epilogue, four warps per 32-lane quarter of TMEM (= 32 rows
+//    of the tile), each taking a quarter of every 64-column chunk.
 //    * bf16 outputs (QKV, FC1+GELU, conv+ReLU) and the fp32 residual stream
-//      (out-proj, FC2): the thread writes its row of a 128-row x 128-byte
-//      chunk into a 128B-swizzled staging buffer in shared memory (bank
-//      conflict free 16-byte stores) and one thread stores the chunk with a
-//      TMA tensor store. For the residual, the old rows of X are brought into
-//      the same staging buffer by TMA loads issued several chunks ahead, so
-//      the read-modify-write of X runs at full memory parallelism.
-//      The 16-bit residual + ReLU of the CNN block outputs works the same way.
+//      (out-proj, FC2): each thread writes its row piece of a 128-row x
+//      128-byte chunk into a 128B-swizzled staging buffer in shared memory
+//      (bank conflict free 16-byte stores) and one thread stores the chunk
+//      with a TMA tensor store. For the residual, the old rows of X are
+//      brought into the same staging buffer by TMA loads issued several
+//      chunks ahead, so the read-modify-write of X runs at full memory
+//      parallelism. The 16-bit residual + ReLU of the CNN block outputs works
+//      the same way.
 //    * the remaining epilogues (fp32 out, patch rows with position
 //      embedding) transpose through padded shared memory for row-contiguous
-//      stores.
+//      stores (warps 2-5); the fp32 one also writes the partial sums of a
+//      split-K plan, whose k-block range is tile / (mt * nt).
+//  - implicit-GEMM convolution: A tiles are 4-D TMA boxes of the NHWC input
+//    (one tap and channel group per k-block, padding read as zeros), and the
+//    output is stored by 4-D boxes of the tile's pixel block.
 //  Every mbarrier wait is bounded; a timeout records ELASTO_ERR_TIMEOUT.
 #include <algorithm>
 
