@@ -11,17 +11,21 @@
 // weights downstream, so the padding changes no output).
 //
 // Forward, all convolutions on the tcgen05 GEMM of gemm.cu:
-//   stem     7x7/2 conv: gather (ky, kx, c) patch rows, GEMM + bias + ReLU,
-//            then 3x3/2 max pool (padding never wins);
+//   stem     7x7/2 conv as a 4x4 stride-1 conv over the space-to-depth
+//            image (2x2 pixel blocks -> 12 channels, padded to 16, with a
+//            zero border): one kernel row of an output pixel is 64
+//            contiguous values, one k-block (gemm_plan_conv_rows); + bias +
+//            ReLU, then 3x3/2 max pool (padding never wins);
 //   block    conv1 1x1: GEMM straight on the NHWC activation [B*H*W, cin];
 //            conv2 3x3/stride: implicit GEMM (gemm_plan_conv): each k-block
-//            (tap, 64 kept channels) is a 4-D TMA tile of the conv1 output,
-//            padding read as zeros, stride by TMA traversal strides; + bias
-//            + ReLU;
+//            (tap, 64 kept channels; 16 when at most 16 are kept) is a 4-D
+//            TMA tile of the conv1 output, padding read as zeros, stride by
+//            TMA traversal strides; + bias + ReLU;
 //            projection (first block of a stage): 1x1/stride conv + bias
 //            (an implicit GEMM too when the stride is 2);
 //            conv3 1x1: GEMM + bias + shortcut + ReLU in the epilogue;
-//   head     global average pool (fp32), classifier in fp32.
+//   head     global average pool (fp32), classifier in fp32 (pooled rows
+//            staged in shared memory).
 //
 // Operands are f16, not bf16: the tensor cores multiply both at the same rate
 // (kind::f16 with f16 A and B, fp32 accumulation), and f16's 11-bit
