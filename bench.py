@@ -98,29 +98,39 @@ class ClockSampler:
             self.proc.wait(timeout=5)
         except Exception:
             self.proc.kill()
-        rows = []
-        for line in open(self.path).read().splitlines():
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) >= 9:
-                rows.append(parts)
+        text = open(self.path).read()
         os.unlink(self.path)
-        if not rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return summarize_clock_rows(text.splitlines())
 
-        def num(x):
-            try:
-                return float(x)
-            except ValueError:
-                return None
-        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
-        smax = [num(r[2]) for r in rows if num(r[2]) is not None]
-        power = [num(r[3]) for r in rows if num(r[3]) is not None]
-        loaded = [s for s, p in zip(sm, power) if p is not None and p > 300] or sm
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
-        return {"sm_mhz": statistics.median(loaded) if loaded else None,
-                "sm_max_mhz": max(smax) if smax else None, "reasons": reasons, "samples": len(rows),
-                "power_w_max": max(power) if power else None}
+
+def summarize_clock_rows(lines):
+    """Clock record from nvidia-smi CSV lines of ClockSampler.QUERY (no header,
+    no units): median SM clock over the samples drawing more than 300 W (all
+    samples if none does), the maximum clock, and every throttle reason seen
+    active."""
+    rows = []
+    for line in lines:
+        parts = [x.strip() for x in line.split(",")]
+        if len(parts) >= 9:
+            rows.append(parts)
+    if not rows:
+        return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+
+    def num(x):
+        try:
+            return float(x)
+        except ValueError:
+            return None
+    samples = [(num(r[1]), num(r[3])) for r in rows]
+    sm = [c for c, _ in samples if c is not None]
+    smax = [num(r[2]) for r in rows if num(r[2]) is not None]
+    power = [p for _, p in samples if p is not None]
+    loaded = [c for c, p in samples if c is not None and p is not None and p > 300] or sm
+    names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+    reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+    return {"sm_mhz": statistics.median(loaded) if loaded else None,
+            "sm_max_mhz": max(smax) if smax else None, "reasons": reasons, "samples": len(rows),
+            "power_w_max": max(power) if power else None}
 
 
 # ---------------------------------------------------------------------------- oracle timing
