@@ -302,13 +302,16 @@ def main():
         return times, per_kind, recs_first
 
     # ------------------------------------------------ headline: full mode, batch B
-    times, per_kind, recs = timed_steps(args.mode, 3, args.warmup)  # warm-up incl. profiler
+    # Timed without the library's per-launch events (they would break the
+    # programmatic-dependent-launch overlap between kernels); the kernel
+    # shares and the roofline come from a profiled pass right after.
+    timed_steps(args.mode, 1, args.warmup, profile=False)
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
     clk = ClockSampler(local)
     clk.start()
-    times, per_kind, recs = timed_steps(args.mode, args.steps, 0)
+    times, _, _ = timed_steps(args.mode, args.steps, 0, profile=False)
     clocks = clk.stop()
     torch.cuda.synchronize()
     if dist:
@@ -318,12 +321,17 @@ def main():
     tflops = 2.0 * macs_img * B * args.steps / (float(sum(times)) / 1e3) / 1e12
     launches = model.query(binding.Q_LAUNCHES, args.mode)
 
+    # profiled pass (same workload, L2 flushed per step): per-launch CUDA
+    # events recorded by the library on the forward's stream
+    prof_steps = max(3, min(args.steps, 20))
+    ptimes, per_kind, recs = timed_steps(args.mode, prof_steps, 2, profile=True)
+
     # dominant kernel: the tcgen05 GEMM (all its launches in the step)
     total_kernel_ms = sum(v[0] for k, v in per_kind.items() if k != "gemm")
     kinds = {}
     for k, v in per_kind.items():
-        e = {"ms_per_step": v[0] / args.steps, "share": v[0] / total_kernel_ms,
-             "launches_per_step": v[3] / args.steps}
+        e = {"ms_per_step": v[0] / prof_steps, "share": v[0] / total_kernel_ms,
+             "launches_per_step": v[3] / prof_steps}
         if v[1] > 0:
             e["tflops"] = 2.0 * v[1] / (v[0] / 1e3) / 1e12
         if k in ("layernorm", "attention", "patchify", "head"):
@@ -331,14 +339,17 @@ def main():
         kinds[k] = e
     g = per_kind.get("gemm", [1e-9, 0, 0, 1])
     gemm_tflops = 2.0 * g[1] / (g[0] / 1e3) / 1e12
-    peak_t = peaks["bf16_tflops_sustained"]
+    peak_t = peaks["bf16_tflops"]
     traffic = committed_traffic("gemm_tc_kernel", os.path.join(ROOT, "paper_2609_10018_gb300", "csrc", "gemm.cu"))
     roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (all epilogues; tcgen05 M=128 tiles)",
                 "achieved": gemm_tflops, "peak": peak_t, "unit": "TFLOP/s", "frac": gemm_tflops / peak_t,
-                "traffic": traffic, "peak_source": f"{peak_src} bf16_tflops_sustained (GEMMs timed inside a "
-                                                   f"{statistics.mean(times):.1f} ms step)",
+                "traffic": traffic,
+                "peak_source": f"{peak_src} bf16_tflops (burst: the GEMMs run inside {prof_steps} steps of "
+                               f"{statistics.mean(ptimes):.1f} ms, a region of {sum(ptimes) / 1e3:.2f} s)",
                 "algorithmic": "2 x M x N x K per launch (kept widths only), summed over the step's GEMM launches",
-                "launches_per_step": g[3] / args.steps, "ms_per_step": g[0] / args.steps}
+                "timing": f"CUDA events around every launch, profiled pass of {prof_steps} steps after the headline",
+                "launches_per_step": g[3] / prof_steps, "ms_per_step": g[0] / prof_steps,
+                "profiled_step_ms": statistics.mean(ptimes)}
 
     line = {"metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,

@@ -169,10 +169,12 @@ elasto_status elasto_forward_host(elasto_t h, void* stream, const void* images_h
  * the handle's own workspace is not used and batch is limited by that array,
  * not by max_batch: a batch whose scratch does not fit is rejected with
  * ELASTO_ERR_INVALID_ARG and a message giving the limit for the model and
- * current mode (e.g. 18 images for the full ViT-B/16 mode, 239 for the tiny ViT).
- * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress) once; make that first call before any stream
- * capture. Every call uses the same array and it keeps the last call's
+ * current mode (e.g. 18 images for the full ViT-B/16 mode, 238 for the tiny ViT).
+ * The current device must be the handle's (else INVALID_ARG). The first call
+ * in a CUDA context of a device looks up the array's device address
+ * (cudaGetSymbolAddress), and the first call for each (mode, batch) builds
+ * its launch plans and keeps them with the handle (host memory); make those
+ * first calls before any stream capture. Every call uses the same array and it keeps the last call's
  * contents; each call writes all the scratch it reads, so nothing has to be
  * cleared, but calls that overlap on the GPU (e.g. on two streams) race on
  * it: order them on one stream. Asynchronous like elasto_forward; images and

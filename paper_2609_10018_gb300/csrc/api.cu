@@ -1064,6 +1064,7 @@ elasto_status elasto_destroy(elasto_t h) {
   cudaDeviceSynchronize();
   if (h->arena) cudaFree(h->arena);
   if (h->cnn) cnn_destroy(h->cnn);
+  noalloc_cache_free(h->noalloc);
   h->prof.release();
   delete h;
   return ELASTO_OK;

@@ -86,7 +86,6 @@ enum GemmEpi : int {
   EPI_BIAS_RELU_F16 = ELASTO_EPI_BIAS_RELU_F16,
   EPI_BIAS_F16 = ELASTO_EPI_BIAS_F16,
   EPI_BIAS_RESID_RELU_F16 = ELASTO_EPI_BIAS_RESID_RELU_F16,
-  EPI_PATCH_POS_F32 = 16,  // patch embedding: out row remapped past the class token, + position embedding
 };
 
 struct GemmArgs {
@@ -95,9 +94,6 @@ struct GemmArgs {
   const float* bias;      // [N] or null
   void* out;              // [*, ldo]
   int ldo;
-  int patches;            // PATCH: patches per image
-  int tokens;             // PATCH: tokens per image (patches + 1)
-  const float* pos;       // PATCH: [tokens, N]
   int* status;
   int stages;             // operand ring depth (<= 8)
   int b_stage;            // bytes of one B stage (both planes; half of B for a CTA pair)
@@ -252,10 +248,6 @@ cudaError_t cnn_init_attributes();
 cudaError_t layernorm_launch(const float* x, const float* g, const float* b, bf16* y, int rows, int d, int d_true,
                              cudaStream_t s);
 cudaError_t softmax_launch(const float* x, float* y, int rows, int cols, cudaStream_t s);
-// images [B, H, W, C] (bf16 or fp32) -> A [B * np, P*P*C] bf16 in (ky, kx, c)
-// order; also writes the class-token rows X[b * n] = cls + pos[0].
-cudaError_t patchify_launch(const void* images, int img_dtype, int B, int H, int W, int C, int P, bf16* A,
-                            float* X, const float* cls, const float* pos, int d, cudaStream_t s);
 // images [B, H, W, C] -> A [B * n, P*P*C] bf16 in token order: row b*n is the
 // class token's slot (zeros), row b*n + 1 + p holds patch p in (ky, kx, c)
 // order. 16-byte copies when the images are bf16 and P*C % 8 == 0.

@@ -216,56 +216,6 @@ cudaError_t softmax_launch(const float* x, float* y, int rows, int cols, cudaStr
 // ---------------------------------------------------------------- patches
 namespace {
 
-// One thread per 2 output elements of A[B * np, P*P*C] ((ky, kx, c) order);
-// the class-token rows are written by the first B * d threads.
-template <typename T>
-__global__ void patchify_kernel(const T* __restrict__ img, int B, int H, int W, int C, int P, bf16* __restrict__ A,
-                                float* __restrict__ X, const float* __restrict__ cls, const float* __restrict__ pos,
-                                int d) {
-  pdl_wait();
-  pdl_trigger();
-  const int gw = W / P, np = (H / P) * gw, K = P * P * C;
-  const size_t total2 = static_cast<size_t>(B) * np * K / 2;
-  const size_t t = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (t < static_cast<size_t>(B) * d) {
-    const int bb = static_cast<int>(t / d), c = static_cast<int>(t % d);
-    X[static_cast<size_t>(bb) * (np + 1) * d + c] = cls[c] + pos[c];
-  }
-  if (t >= total2) return;
-  float v[2];
-#pragma unroll
-  for (int e = 0; e < 2; ++e) {
-    const size_t idx = 2 * t + e;
-    const int k = static_cast<int>(idx % K);
-    const size_t row = idx / K;
-    const int p = static_cast<int>(row % np), bb = static_cast<int>(row / np);
-    const int c = k % C, kx = (k / C) % P, ky = k / (C * P);
-    const int yy = (p / gw) * P + ky, xx = (p % gw) * P + kx;
-    const T val = img[((static_cast<size_t>(bb) * H + yy) * W + xx) * C + c];
-    if constexpr (sizeof(T) == 2)
-      v[e] = __bfloat162float(val);
-    else
-      v[e] = static_cast<float>(val);
-  }
-  reinterpret_cast<uint32_t*>(A)[t] = pack_bf16x2(v[0], v[1]);
-}
-
-}  // namespace
-
-cudaError_t patchify_launch(const void* images, int img_dtype, int B, int H, int W, int C, int P, bf16* A, float* X,
-                            const float* cls, const float* pos, int d, cudaStream_t s) {
-  const size_t total2 = static_cast<size_t>(B) * (H / P) * (W / P) * P * P * C / 2;
-  const size_t threads = total2 > static_cast<size_t>(B) * d ? total2 : static_cast<size_t>(B) * d;
-  const unsigned blocks = static_cast<unsigned>((threads + 255) / 256);
-  if (img_dtype == ELASTO_BF16)
-    return launch_pdl(patchify_kernel<bf16>, dim3(blocks), dim3(256), 0, s, static_cast<const bf16*>(images), B, H, W,
-                      C, P, A, X, cls, pos, d);
-  return launch_pdl(patchify_kernel<float>, dim3(blocks), dim3(256), 0, s, static_cast<const float*>(images), B, H,
-                    W, C, P, A, X, cls, pos, d);
-}
-
-namespace {
-
 // A [B * n, K] in token order, K = P*P*C in (ky, kx, c) order. One thread per
 // 16-byte piece (8 bf16): within a patch row, the P*C values (kx, c) are
 // contiguous in the NHWC image, so a piece is one aligned 16-byte copy.

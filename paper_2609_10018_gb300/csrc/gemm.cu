@@ -29,10 +29,10 @@
 //      chunks ahead, so the read-modify-write of X runs at full memory
 //      parallelism. The 16-bit residual + ReLU of the CNN block outputs works
 //      the same way.
-//    * the remaining epilogues (fp32 out, patch rows with position
-//      embedding) transpose through padded shared memory for row-contiguous
-//      stores (warps 2-5); the fp32 one also writes the partial sums of a
-//      split-K plan, whose k-block range is tile / (mt * nt).
+//    * the remaining epilogue (fp32 out) transposes through padded shared
+//      memory for row-contiguous stores (warps 2-5); it also writes the
+//      partial sums of a split-K plan, whose k-block range is
+//      tile / (mt * nt).
 //  - implicit-GEMM convolution: A tiles are 4-D TMA boxes of the NHWC input
 //    (one tap and channel group per k-block, padding read as zeros), and the
 //    output is stored by 4-D boxes of the tile's pixel block.
@@ -636,28 +636,15 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
         for (int j = 0; j < 32; ++j) st[lane * EPI_LD + j] = __uint_as_float(r[j]);
         __syncwarp();
-        {  // EPI_BIAS_F32 or EPI_PATCH_POS_F32
+        {  // EPI_BIAS_F32
           const int col = n0 + c + lane;
           const bool cok = col < N;
           const float bv = (cok && args.bias) ? args.bias[col] : 0.0f;
           float* out = static_cast<float*>(args.out) + (t / mn_tiles) * args.split_stride;
-          if constexpr (EPI == EPI_BIAS_F32) {
 #pragma unroll 8
-            for (int i = 0; i < 32; ++i) {
-              const int row = row0 + i;
-              if (cok && row < M) out[static_cast<size_t>(row) * args.ldo + col] = st[i * EPI_LD + lane] + bv;
-            }
-          } else {
-#pragma unroll 8
-            for (int i = 0; i < 32; ++i) {
-              const int row = row0 + i;
-              if (cok && row < M) {
-                const int img = row / args.patches, p = row - img * args.patches;
-                const size_t orow = static_cast<size_t>(img) * args.tokens + 1 + p;
-                out[orow * args.ldo + col] =
-                    (st[i * EPI_LD + lane] + bv) + args.pos[static_cast<size_t>(1 + p) * N + col];
-              }
-            }
+          for (int i = 0; i < 32; ++i) {
+            const int row = row0 + i;
+            if (cok && row < M) out[static_cast<size_t>(row) * args.ldo + col] = st[i * EPI_LD + lane] + bv;
           }
         }
         __syncwarp();
@@ -830,7 +817,6 @@ cudaError_t gemm_init_attributes() {
   SET_ATTR(EPI_BIAS_F32)
   SET_ATTR(EPI_BIAS_RELU_BF16)
   SET_ATTR(EPI_BIAS_RESID_RELU_BF16)
-  SET_ATTR(EPI_PATCH_POS_F32)
   SET_ATTR(EPI_BIAS_RELU_F16)
   SET_ATTR(EPI_BIAS_F16)
   SET_ATTR(EPI_BIAS_RESID_RELU_F16)
@@ -1188,7 +1174,6 @@ cudaError_t gemm_launch_main(const GemmPlan& p, int M, cudaStream_t s) {
     CASE(EPI_BIAS_F32)
     CASE_PAIR(EPI_BIAS_RELU_BF16)
     CASE(EPI_BIAS_RESID_RELU_BF16)
-    CASE(EPI_PATCH_POS_F32)
     CASE_PAIR(EPI_BIAS_RELU_F16)
     CASE_PAIR(EPI_BIAS_F16)
     CASE(EPI_BIAS_RESID_RELU_F16)

@@ -43,6 +43,11 @@ struct VitEmbed {
   GemmPlanSet patch;        // pruned modes: the patch projection at width d_pad
 };
 
+// Launch plans of elasto_forward_noalloc (csrc/noalloc.cu), cached per
+// (mode, batch); host memory only.
+struct NoallocCache;
+void noalloc_cache_free(NoallocCache* c);
+
 struct VitMode {
   std::vector<VitLayerPack> layers;
   VitEmbed emb;
@@ -88,6 +93,7 @@ struct elasto_s {
   std::vector<std::vector<int32_t>> perm_h, perm_f;
   size_t packed_total = 0;  // device bytes of all modes' packed weights
   std::atomic<int> cur{0};
+  elasto::NoallocCache* noalloc = nullptr;  // built by the first elasto_forward_noalloc call
   // CNN state lives behind this pointer (null for ViT)
   elasto::CnnModel* cnn = nullptr;
   elasto::Profiler prof;

@@ -40,3 +40,37 @@ def margin(ref: np.ndarray) -> np.ndarray:
     """Oracle top-1 minus top-2 logit, per image."""
     s = np.sort(ref, axis=1)
     return s[:, -1] - s[:, -2]
+
+
+CENTERED_TOL = 2e-2  # on the image-dependent part of the logits alone
+
+
+def centered(x: np.ndarray) -> np.ndarray:
+    """Logits minus their mean over the batch: the part that varies from image
+    to image."""
+    return x - x.mean(axis=0, keepdims=True)
+
+
+def check_image_dependent_part(tag: str, got: np.ndarray, ref: np.ndarray) -> dict:
+    """With random weights most of a logit is the same for every image (the
+    ViTs give every image the same top class), so besides max|dlogit| this
+    checks the part that the images themselves decide: the centred logits
+    within CENTERED_TOL, and the top class of the centred logits the same as
+    the oracle's wherever the oracle's own centred margin exceeds twice the
+    largest centred error (where it does not, either class is a valid
+    answer)."""
+    cg, cr = centered(got), centered(ref)
+    cerr = rel_err(cg, cr)
+    dmax = float(np.max(np.abs(cg - cr)))
+    cm = margin(cr)
+    decided = cm > 2.0 * dmax
+    agree_c = cg.argmax(axis=1) == cr.argmax(axis=1)
+    out = {"err": rel_err(got, ref), "top1": top1_agreement(got, ref), "centred_err": cerr,
+           "centred_share": float(np.max(np.abs(cr)) / np.max(np.abs(ref))),
+           "centred_top1": float(np.mean(agree_c)), "centred_decided": int(decided.sum())}
+    print(f"{tag}: err {out['err']:.2e} top1 {out['top1']:.4f} | image-dependent part "
+          f"{out['centred_share']:.2e} of max|logit|, its err {cerr:.2e}, centred top-1 "
+          f"{out['centred_top1']:.4f} ({out['centred_decided']}/{len(ref)} decided by margin)")
+    assert cerr <= CENTERED_TOL, (tag, cerr)
+    assert np.all(agree_c[decided]), (tag, np.flatnonzero(decided & ~agree_c))
+    return out

@@ -67,9 +67,10 @@ def test_resnet50_small_all_modes_2000_images():
 
 
 def test_resnet50_224_all_modes():
+    """224x224 (ImageNet-shaped), 64 images per mode."""
     cfg = synth.RESNET50
     w, tables = synth.make_resnet_weights(cfg), synth.make_resnet_tables(cfg)
-    n_img = 16
+    n_img = 64
     img = synth.make_images(cfg, n_img)
     with binding.ElasticModel.resnet(cfg, w, tables, max_batch=n_img) as model:
         x = dev(img)
@@ -78,7 +79,8 @@ def test_resnet50_224_all_modes():
             ref = resnet_logits(cfg, tables, m, img, chunk=2)
             err, agree = _report(f"resnet50 224px mode {m}", got, ref)
             assert err <= TOL
-            assert agree == 1.0
+            decided = margin(ref) > 2.0 * float(np.max(np.abs(got - ref)))
+            assert np.all((got.argmax(axis=1) == ref.argmax(axis=1)) | ~decided)
 
 
 def test_resnet_packed_weights_match_oracle_folding():

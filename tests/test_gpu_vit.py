@@ -3,12 +3,17 @@ fp64 oracle: every mode of the tiny, ViT-S/16 and ViT-B/16 configurations,
 bit-exact packed layouts, mode switching, degenerate tables.
 
 Acceptance (per mode): max|dlogit| <= 1e-2 * max|logit_oracle|, and top-1
-agreement >= 99.9 % where the image count makes that meaningful (2000 tiny
-images per mode); at ViT-S/B sizes the oracle checks sampled images."""
+agreement >= 99.9 % (2000 tiny images per mode, 256 ViT-S/16 images per mode,
+all 256 images of a ViT-B/16 batch in the full and smallest mode). With
+random weights the ViTs give almost every image the same top class, so the
+image-dependent part of the logits (centred over the batch) is checked as
+well: within 2e-2, and its top class equal to the oracle's wherever the
+oracle's margin decides it."""
 import numpy as np
 import pytest
 
-from helpers import dev, empty_dev, margin, rel_err, stream_handle, top1_agreement
+from helpers import check_image_dependent_part, dev, empty_dev, margin, rel_err, stream_handle, top1_agreement
+from oracle_pool import vit_logits
 from oracle import vit as ov
 from paper_2609_10018_gb300 import binding, synth
 
@@ -49,6 +54,7 @@ def test_tiny_all_modes_2000_images(tiny):
                   f"{np.median(mg):.3e}")
             assert err <= TOL
             assert agree >= 0.999
+            check_image_dependent_part(f"tiny mode {m} ({n_img} images)", got, ref)
 
 
 def test_tiny_batch_8_matches_oracle(tiny):
@@ -75,35 +81,60 @@ def test_packed_layouts_bit_exact(cfg):
                     assert out.tobytes() == ref[name].tobytes(), (m, l, name)
 
 
+def _check_top1(tag, got, ref):
+    """Top-1 agreement >= 99.9 %, where a disagreement only counts if the
+    oracle's own top-1/top-2 margin exceeds twice the largest logit error
+    (below that either class is a valid answer)."""
+    agree = got.argmax(axis=1) == ref.argmax(axis=1)
+    decided = margin(ref) > 2.0 * float(np.max(np.abs(got - ref)))
+    assert np.mean(agree | ~decided) >= 0.999, (tag, np.flatnonzero(decided & ~agree))
+
+
+def _parity_rows(cfg, tag, got, ref):
+    out = check_image_dependent_part(tag, got, ref)
+    assert out["err"] <= TOL, (tag, out["err"])
+    _check_top1(tag, got, ref)
+    assert np.all(np.isfinite(got))
+
+
 def _sampled_parity(cfg, batch, sample, modes=None):
     w = synth.make_vit_weights(cfg)
-    wide = ov.widen_all(w)
     tables = synth.make_vit_tables(cfg)
     img = synth.make_images(cfg, batch)
     with binding.ElasticModel.vit(cfg, w, tables, max_batch=batch) as model:
         x = dev(img)
         for m in (modes if modes is not None else range(len(tables))):
-            t = tables[m]
+            rows = sample(m) if callable(sample) else sample
             got = _run(model, x, batch, cfg.classes, m)
-            ref = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img[sample])
-            err = rel_err(got[sample], ref)
-            print(f"{cfg.name} B={batch} mode {m}: err {err:.2e}, top-1 {top1_agreement(got[sample], ref):.3f}")
-            assert err <= TOL
-            assert top1_agreement(got[sample], ref) == 1.0 or np.min(margin(ref)) < 2 * TOL * np.max(np.abs(ref))
-            assert np.all(np.isfinite(got))
+            ref = vit_logits(cfg, tables, m, img[rows])
+            _parity_rows(cfg, f"{cfg.name} B={batch} mode {m} ({len(rows)} images)", got[rows], ref)
 
 
-def test_vit_s_batch_64_all_modes():
-    _sampled_parity(synth.VIT_S, 64, np.array([0, 1, 31, 62, 63]))
+def test_vit_s_256_images_all_modes():
+    """ViT-S/16 at its batch of 64: four batches, 256 images per mode, every
+    one against the oracle."""
+    cfg = synth.VIT_S
+    w = synth.make_vit_weights(cfg)
+    tables = synth.make_vit_tables(cfg)
+    n_img, B = 256, cfg.batch
+    img = synth.make_images(cfg, n_img)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=B) as model:
+        for m in range(len(tables)):
+            got = np.concatenate([_run(model, dev(img[i:i + B]), B, cfg.classes, m) for i in range(0, n_img, B)])
+            ref = vit_logits(cfg, tables, m, img)
+            _parity_rows(cfg, f"{cfg.name} mode {m} ({n_img} images)", got, ref)
 
 
 def test_vit_b_batch_256_all_modes():
-    _sampled_parity(synth.VIT_B, 256, np.array([0, 97, 254, 255]))
+    """ViT-B/16 at batch 256: all 256 images of the full and the smallest mode,
+    every eighth image (32) of the others."""
+    last = len(synth.VIT_B.mode_heads) - 1
+    _sampled_parity(synth.VIT_B, 256, lambda m: np.arange(256) if m in (0, last) else np.arange(0, 256, 8))
 
 
 @pytest.mark.parametrize("batch", [1, 32])
 def test_vit_b_small_batches(batch):
-    _sampled_parity(synth.VIT_B, batch, np.array([0, batch - 1]), modes=[0, 4])
+    _sampled_parity(synth.VIT_B, batch, np.arange(batch), modes=[0, 4])
 
 
 def test_one_image_on_larger_handles_all_modes(tiny):

@@ -251,3 +251,56 @@ def test_pack_rounds_fp32_to_nearest_even():
     # 1+3*2^-8 is a tie between 1+2^-7 and 1+2^-6 -> even (1+2^-6)
     assert back.tolist() == [1.0, 1.0, 1.0 + 2**-7, 1.0 + 2**-6, -2.5, 1.0]
     assert np.array_equal(bits, torch.from_numpy(vals).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16))
+
+
+# ---------------------------------------------------------------- input widening
+
+def _bf16_by_definition(bits: int) -> float:
+    """Value of a bf16 bit pattern from the format's fields: 1 sign bit, 8
+    exponent bits (bias 127), 7 fraction bits; exponent 0 is subnormal
+    (2^-126 * f / 128), exponent 255 is infinity (f = 0) or NaN."""
+    import math
+    s, e, f = bits >> 15, (bits >> 7) & 0xFF, bits & 0x7F
+    sign = -1.0 if s else 1.0
+    if e == 0xFF:
+        return sign * math.inf if f == 0 else math.nan
+    if e == 0:
+        return sign * math.ldexp(f, -126 - 7)
+    return sign * math.ldexp(128 + f, e - 127 - 7)
+
+
+def test_widen_decodes_every_bf16_pattern():
+    """oracle.vit.widen on all 65,536 bf16 bit patterns against (a) the format's
+    field definition and (b) torch's own bfloat16 -> float64 conversion; NaNs
+    compare as NaN, and the sign of zero is kept. A wrong shift, byte order or
+    sign handling fails here."""
+    bits = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    got = ov.widen(bits)
+    assert got.dtype == np.float64 and got.shape == (65536,)
+    by_def = np.array([_bf16_by_definition(int(b)) for b in range(65536)])
+    lib = torch.from_numpy(bits.view(np.int16).copy()).view(torch.bfloat16).to(torch.float64).numpy()
+    for ref in (by_def, lib):
+        nan = np.isnan(ref)
+        assert np.array_equal(np.isnan(got), nan)
+        assert np.array_equal(got[~nan], ref[~nan])
+        assert np.array_equal(np.signbit(got[~nan]), np.signbit(ref[~nan]))
+    # a few patterns worked out by hand
+    hand = {0x3F80: 1.0, 0x4000: 2.0, 0xC040: -3.0, 0x3F81: 1.0 + 2.0**-7, 0x0001: 2.0**-133,
+            0x0080: 2.0**-126, 0x7F7F: (2.0 - 2.0**-7) * 2.0**127, 0x7F80: np.inf, 0xFF80: -np.inf,
+            0x3E80: 0.25, 0xBF00: -0.5}
+    for b, v in hand.items():
+        assert got[b] == v, hex(b)
+    assert np.isnan(got[0x7FC0]) and got[0x8000] == 0.0 and np.signbit(got[0x8000])
+
+
+def test_widen_keeps_fp32_and_multidimensional_arrays_exact():
+    """fp32 inputs widen to the same real number, and bf16 arrays keep their
+    shape and element order (a transposed or flattened decode fails)."""
+    rng = np.random.default_rng(5)
+    f = rng.standard_normal((3, 5)).astype(np.float32)
+    assert np.array_equal(ov.widen(f), f.astype(np.float64)) and ov.widen(f).dtype == np.float64
+    b = rng.integers(0, 0x7F80, size=(4, 3, 2)).astype(np.uint16)  # finite positives
+    got = ov.widen(b)
+    assert got.shape == b.shape
+    for idx in np.ndindex(b.shape):
+        assert got[idx] == _bf16_by_definition(int(b[idx]))

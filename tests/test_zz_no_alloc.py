@@ -6,12 +6,14 @@ synchronisation an allocation may cause). Its activations live in a fixed
 
 Checked here, through the C-ABI: on two calls in a row its logits match
 elasto_forward's on the same inputs within the parity tolerance the other
-tests use, and a batch whose scratch does not fit in the array is rejected
-with a clear error. This file is collected last on purpose."""
+tests use, and the fp64 oracle's directly; the device's free memory does not
+change across calls; and a batch whose scratch does not fit in the array is
+rejected with a clear error. This file is collected last on purpose."""
 import numpy as np
 import pytest
 
 from helpers import dev, empty_dev, rel_err, stream_handle
+from oracle import vit as ov
 from paper_2609_10018_gb300 import binding, synth
 
 pytestmark = pytest.mark.gpu
@@ -34,16 +36,47 @@ def _logits_both_ways(model, cfg, images, batch, mode):
     return ref.cpu().numpy().astype(np.float64), [o.cpu().numpy().astype(np.float64) for o in outs]
 
 
-def test_noalloc_matches_forward_tiny_all_modes():
+def test_noalloc_matches_forward_and_oracle_tiny_all_modes():
+    cfg = synth.TINY
+    w = synth.make_vit_weights(cfg)
+    wide = ov.widen_all(w)
+    tables = synth.make_vit_tables(cfg)
+    img = synth.make_images(cfg, cfg.batch)
+    images = dev(img)
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=cfg.batch) as model:
+        for m, t in enumerate(tables):
+            ref, outs = _logits_both_ways(model, cfg, images, cfg.batch, m)
+            want = ov.vit_forward_sliced(wide, cfg, t["heads"], t["mlp"], img)
+            for o in outs:
+                assert rel_err(o, ref) <= TOL
+                assert rel_err(o, want) <= TOL
+
+
+def test_noalloc_leaves_free_device_memory_unchanged():
+    """After a first call (which looks up the array's address and builds the
+    launch plans), further calls change the device's free memory by nothing:
+    they allocate no device memory."""
+    import torch
     cfg = synth.TINY
     w = synth.make_vit_weights(cfg)
     tables = synth.make_vit_tables(cfg)
-    images = dev(synth.make_images(cfg, cfg.batch))
-    with binding.ElasticModel.vit(cfg, w, tables, max_batch=cfg.batch) as model:
+    B = 32  # beyond max_batch: the handle's workspace could not hold it
+    images = dev(synth.make_images(cfg, B))
+    out = empty_dev((B, cfg.classes), torch.float32)
+    s = stream_handle()
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=1) as model:
         for m in range(len(tables)):
-            ref, outs = _logits_both_ways(model, cfg, images, cfg.batch, m)
-            for o in outs:
-                assert rel_err(o, ref) <= TOL
+            model.set_mode(m)
+            binding.elasto_forward_noalloc(model.handle, s, images.data_ptr(), B, out.data_ptr())
+        model.sync_status(s)
+        free0, _ = torch.cuda.mem_get_info()
+        for _ in range(3):
+            for m in range(len(tables)):
+                model.set_mode(m)
+                binding.elasto_forward_noalloc(model.handle, s, images.data_ptr(), B, out.data_ptr())
+        model.sync_status(s)
+        free1, _ = torch.cuda.mem_get_info()
+        assert free1 == free0
 
 
 def test_noalloc_vit_b_largest_batch_and_limit():
