@@ -54,7 +54,7 @@ def test_tiny_all_modes_2000_images(tiny):
                   f"{np.median(mg):.3e}")
             assert err <= TOL
             assert agree >= 0.999
-            check_image_dependent_part(f"tiny mode {m} ({n_img} images)", got, ref)
+            check_image_dependent_part(f"tiny mode {m} ({n_img} images)", got, ref, cfg.layers)
 
 
 def test_tiny_batch_8_matches_oracle(tiny):
@@ -91,7 +91,7 @@ def _check_top1(tag, got, ref):
 
 
 def _parity_rows(cfg, tag, got, ref):
-    out = check_image_dependent_part(tag, got, ref)
+    out = check_image_dependent_part(tag, got, ref, cfg.layers)
     assert out["err"] <= TOL, (tag, out["err"])
     _check_top1(tag, got, ref)
     assert np.all(np.isfinite(got))
