@@ -150,7 +150,10 @@ def test_softmax_matches_fp64(rows, cols):
     assert np.allclose(got.sum(1), 1.0, atol=1e-5)
 
 
-ATTN_CASES = [(2, 197, 3), (3, 65, 2), (1, 256, 1), (2, 1, 1), (2, 17, 4), (1, 129, 12)]
+# the last three give each of the 152 persistent CTAs four or more items, so
+# every K/V slot and Q buffer is reused (2 slots at n = 256, 3 below 209 keys)
+ATTN_CASES = [(2, 197, 3), (3, 65, 2), (1, 256, 1), (2, 1, 1), (2, 17, 4), (1, 129, 12),
+              (160, 256, 4), (120, 65, 6), (100, 129, 7), (64, 197, 12)]
 
 
 @pytest.mark.parametrize("B,n,h", ATTN_CASES)
