@@ -42,7 +42,8 @@ typedef enum {
   ELASTO_ERR_OOM = -4,         /* device allocation failed */
   ELASTO_ERR_CUDA = -5,        /* CUDA runtime/driver error */
   ELASTO_ERR_UNSUPPORTED = -6, /* shape or device the kernels do not support */
-  ELASTO_ERR_TIMEOUT = -7      /* a device-side wait gave up (status word) */
+  ELASTO_ERR_TIMEOUT = -7,     /* a device-side wait gave up (status word) */
+  ELASTO_ERR_GUARD = -8        /* a guard zone after a device buffer was overwritten */
 } elasto_status;
 
 enum { ELASTO_ARCH_VIT = 1, ELASTO_ARCH_RESNET50 = 2 };
@@ -188,6 +189,24 @@ elasto_status elasto_forward_noalloc(elasto_t h, void* stream, const void* image
  * recorded status or ELASTO_OK. */
 elasto_status elasto_sync_status(elasto_t h, void* stream);
 
+/* Out-of-bounds write detection (the paper has no counterpart; a check the
+ * tests run in place of a device memory checker). Every buffer of a handle's
+ * device arena (packed weights, parameters, activations, staging, status
+ * word) is followed by a guard zone of at least 1 KiB, filled with the byte
+ * 0xA5 when the arena is allocated, before any create-time kernel runs.
+ * elasto_check_guards enqueues a check of every zone on `stream`, waits for
+ * it, and returns ELASTO_OK if every guard byte is intact, else
+ * ELASTO_ERR_GUARD with the first damaged zone's buffer named in
+ * elasto_last_error. n_bad (may be null) receives the number of damaged
+ * zones. Errors: INVALID_ARG, CUDA. */
+elasto_status elasto_check_guards(elasto_t h, void* stream, int* n_bad);
+
+/* Test-only: overwrite the first byte of guard zone `zone` (0 <= zone <
+ * elasto_query(ELASTO_Q_GUARD_ZONES)) with a cudaMemset inside the handle's
+ * own allocation, so that a test can see elasto_check_guards report it.
+ * Synchronous. Errors: INVALID_ARG, CUDA. */
+elasto_status elasto_debug_damage_guard(elasto_t h, int zone);
+
 /* Release everything the handle owns (synchronises the device first). */
 elasto_status elasto_destroy(elasto_t h);
 
@@ -207,7 +226,8 @@ enum {
                                     split-K, their partial-sum launches compute the LayerNorms
                                     that follow, and the last FC2's sum stands alone) */
   ELASTO_Q_PACKED_TOTAL = 7,     /* device bytes of all modes' packed weights together */
-  ELASTO_Q_PREFIX_SHARED = 8     /* 1 if the modes share one prefix-ordered packed copy */
+  ELASTO_Q_PREFIX_SHARED = 8,    /* 1 if the modes share one prefix-ordered packed copy */
+  ELASTO_Q_GUARD_ZONES = 9       /* guard zones in the handle's arena (elasto_check_guards) */
 };
 elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value);
 

@@ -20,10 +20,10 @@ LIB_PATH = os.path.join(_HERE, "libelasto.so")
 
 ARCH_VIT, ARCH_RESNET50 = 1, 2
 F32, BF16 = 0, 1
-OK, ERR_INVALID_ARG, ERR_BAD_TABLE, ERR_BAD_MODE, ERR_OOM, ERR_CUDA, ERR_UNSUPPORTED, ERR_TIMEOUT = (
-    0, -1, -2, -3, -4, -5, -6, -7)
+OK, ERR_INVALID_ARG, ERR_BAD_TABLE, ERR_BAD_MODE, ERR_OOM, ERR_CUDA, ERR_UNSUPPORTED, ERR_TIMEOUT, ERR_GUARD = (
+    0, -1, -2, -3, -4, -5, -6, -7, -8)
 Q_N_MODES, Q_PACKED_BYTES, Q_SHARED_BYTES, Q_WORKSPACE_BYTES, Q_ARENA_BYTES, Q_MODE_MACS, Q_LAUNCHES = range(7)
-Q_PACKED_TOTAL, Q_PREFIX_SHARED = 7, 8
+Q_PACKED_TOTAL, Q_PREFIX_SHARED, Q_GUARD_ZONES = 7, 8, 9
 EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_BIAS_RESID_F32, EPI_BIAS_F32, EPI_BIAS_RELU_BF16, EPI_BIAS_RESID_RELU_BF16 = range(6)
 EPI_BIAS_RELU_F16, EPI_BIAS_F16, EPI_BIAS_RESID_RELU_F16 = range(6, 9)  # A, W, resid, out in IEEE f16
 
@@ -88,6 +88,8 @@ def lib() -> ctypes.CDLL:
         "elasto_forward_host": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
         "elasto_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
         "elasto_sync_status": [c_void_p, c_void_p],
+        "elasto_check_guards": [c_void_p, c_void_p, ctypes.POINTER(c_int)],
+        "elasto_debug_damage_guard": [c_void_p, c_int],
         "elasto_destroy": [c_void_p],
         "elasto_query": [c_void_p, c_int, c_int, ctypes.POINTER(c_int64)],
         "elasto_debug_export_packed": [c_void_p, c_int, c_int, c_int, c_void_p, c_size_t],
@@ -235,6 +237,17 @@ def elasto_forward_host(h: int, stream: int, images: np.ndarray, batch: int, log
 
 def elasto_sync_status(h: int, stream: int = 0) -> None:
     _check(lib().elasto_sync_status(h, stream), "elasto_sync_status")
+
+
+def elasto_check_guards(h: int, stream: int = 0) -> int:
+    """Number of damaged guard zones; raises ElastoError (ERR_GUARD) if any."""
+    n = c_int(0)
+    _check(lib().elasto_check_guards(h, stream, ctypes.byref(n)), "elasto_check_guards")
+    return n.value
+
+
+def elasto_debug_damage_guard(h: int, zone: int) -> None:
+    _check(lib().elasto_debug_damage_guard(h, zone), "elasto_debug_damage_guard")
 
 
 def elasto_destroy(h: int) -> None:
@@ -406,6 +419,11 @@ class ElasticModel:
     def sync_status(self, stream: int = 0) -> None:
         elasto_sync_status(self.handle, stream)
 
+    def check_guards(self, stream: int = 0) -> None:
+        """Raise ElastoError (ERR_GUARD) if any kernel wrote past the end of
+        one of the handle's device buffers."""
+        elasto_check_guards(self.handle, stream)
+
     def query(self, what: int, mode: int = 0) -> int:
         return elasto_query(self.handle, what, mode)
 
@@ -435,5 +453,11 @@ class ElasticModel:
     def __enter__(self):
         return self
 
-    def __exit__(self, *exc):
-        self.close()
+    def __exit__(self, exc_type, exc, tb):
+        # a `with` block that ended normally also proves that no kernel wrote
+        # past the end of a buffer of this handle
+        try:
+            if exc_type is None and self.handle:
+                self.check_guards()
+        finally:
+            self.close()

@@ -31,16 +31,6 @@ namespace {
 
 constexpr size_t kAlign = 1024;
 
-struct Bump {
-  size_t off = 0;
-  size_t take(size_t bytes) {
-    off = (off + kAlign - 1) / kAlign * kAlign;
-    const size_t r = off;
-    off += bytes;
-    return r;
-  }
-};
-
 size_t dtype_size(int dt) { return dt == ELASTO_BF16 ? 2 : 4; }
 
 bool tables_ok(const int32_t* idx, int n, int limit) {
@@ -263,14 +253,14 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   h->kpe = kpe;
 
   // ---------------------------------------------------------------- layout
-  Bump bump;
-  const size_t o_patch_w = bump.take(size_t(D) * kpe * 2);
+  GuardedArena& bump = h->guards;  // every buffer followed by a guard zone
+  const size_t o_patch_w = bump.take(size_t(D) * kpe * 2, "patch projection weights");
   const size_t o_patch_b = bump.take(D * 4), o_cls = bump.take(D * 4), o_pos = bump.take(size_t(n) * D * 4);
   std::vector<size_t> o_l(6 * L);
   for (int l = 0; l < L; ++l)
     for (int k = 0; k < 6; ++k) o_l[6 * l + k] = bump.take(D * 4);
   const size_t o_norm_w = bump.take(D * 4), o_norm_b = bump.take(D * 4);
-  const size_t o_head_w = bump.take(size_t(C) * D * 4), o_head_b = bump.take(C * 4);
+  const size_t o_head_w = bump.take(size_t(C) * D * 4, "classifier weights"), o_head_b = bump.take(C * 4, "classifier bias");
   h->shared_bytes = bump.off;
 
   h->modes.assign(n_modes, VitMode{});
@@ -325,12 +315,12 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
     for (int l = 0; l < L; ++l) {
       const size_t hw = 64 * h->perm_h[l].size(), ff = h->perm_f[l].size();
       SharedOff& o = soff[l];
-      o.qkv_w = bump.take(3 * hw * D * 2);
+      o.qkv_w = bump.take(3 * hw * D * 2, "packed W_qkv");
       o.qkv_b = bump.take(3 * hw * 4);
-      o.proj_w = bump.take(size_t(D) * hw * 2);
-      o.fc1_w = bump.take(ff * D * 2);
+      o.proj_w = bump.take(size_t(D) * hw * 2, "packed W_o");
+      o.fc1_w = bump.take(ff * D * 2, "packed W1");
       o.fc1_b = bump.take(ff * 4);
-      o.fc2_w = bump.take(size_t(D) * ff * 2);
+      o.fc2_w = bump.take(size_t(D) * ff * 2, "packed W2");
       if (split) {
         o.qkv_lo = bump.take(3 * hw * D * 2);
         o.proj_lo = bump.take(size_t(D) * hw * 2);
@@ -400,18 +390,19 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   const size_t o_patch_lo = split ? bump.take(size_t(D) * kpe * 2) : 0;
   const size_t ws_start = bump.off;
   const size_t rows = size_t(Bm) * n;
-  const size_t o_X = bump.take(rows * D * 4), o_Y = bump.take(rows * D * 2);
-  const size_t o_QKV = bump.take(rows * 3 * std::max(wmax, 64) * 2), o_O = bump.take(rows * std::max(wmax, 64) * 2);
-  const size_t o_H = bump.take(rows * std::max(fmax, 8) * 2), o_P = bump.take(rows * kpe * 2);
+  const size_t o_X = bump.take(rows * D * 4, "residual stream X"), o_Y = bump.take(rows * D * 2, "LayerNorm output Y");
+  const size_t o_QKV = bump.take(rows * 3 * std::max(wmax, 64) * 2, "QKV"),
+               o_O = bump.take(rows * std::max(wmax, 64) * 2, "attention output O");
+  const size_t o_H = bump.take(rows * std::max(fmax, 8) * 2, "MLP hidden H"), o_P = bump.take(rows * kpe * 2, "patch rows P");
   // per-token addend of the patch projection: periodic in the token index, so
   // k images' worth (k * n >= n + 128 rows) serve every batch
   h->addend_rows = (1 + (128 + n - 1) / n) * n;
-  const size_t o_tok = bump.take(size_t(h->addend_rows) * D * 4);
+  const size_t o_tok = bump.take(size_t(h->addend_rows) * D * 4, "patch token addend");
   // split-K partial sums of the one-image FC2 (kSplitMax x n x D fp32)
-  const size_t o_part = bump.take(size_t(kSplitMax) * n * D * 4);
+  const size_t o_part = bump.take(size_t(kSplitMax) * n * D * 4, "split-K partial sums");
   const size_t img_bytes = size_t(Bm) * d->img_h * d->img_w * d->img_c * dtype_size(d->weight_dtype);
-  const size_t o_img = bump.take(img_bytes), o_logit = bump.take(size_t(Bm) * C * 4);
-  const size_t o_status = bump.take(64);
+  const size_t o_img = bump.take(img_bytes, "image staging"), o_logit = bump.take(size_t(Bm) * C * 4, "logit staging");
+  const size_t o_status = bump.take(64, "status word");
   h->workspace_bytes = bump.off - ws_start;
   h->arena_bytes = bump.off;
 
@@ -523,6 +514,12 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       }
     }
   ELASTO_CUDA_TRY(cudaMemset(h->arena, 0, h->arena_bytes));
+  {
+    // guard zones filled right after the arena is cleared, before any
+    // create-time kernel writes to it, so that those are checked too
+    const elasto_status gs = h->guards.upload(h->arena);
+    if (gs != ELASTO_OK) return gs;
+  }
 
   // ---------------------------------------------------------------- upload
   const int dt = d->weight_dtype;
@@ -972,6 +969,7 @@ elasto_status elasto_create(const elasto_model_desc* desc, const elasto_weights*
   if (st != ELASTO_OK) {
     cudaDeviceSynchronize();
     if (h->arena) cudaFree(h->arena);
+    h->guards.release();
     if (h->cnn) cnn_destroy(h->cnn);
     return st;
   }
@@ -1065,12 +1063,53 @@ elasto_status elasto_destroy(elasto_t h) {
   if (h->arena) cudaFree(h->arena);
   if (h->cnn) cnn_destroy(h->cnn);
   noalloc_cache_free(h->noalloc);
+  h->guards.release();
   h->prof.release();
   delete h;
   return ELASTO_OK;
 }
 
 const char* elasto_last_error(void) { return last_error_cstr(); }
+
+elasto_status elasto_check_guards(elasto_t h, void* stream, int* n_bad) {
+  if (!h) {
+    set_error("elasto_check_guards: null handle");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  char* base = h->arena;
+  GuardedArena* g = &h->guards;
+  if (h->cnn) g = cnn_guards(h->cnn, &base);
+  std::string first;
+  const int bad = g->check(base, static_cast<cudaStream_t>(stream), &first);
+  if (n_bad) *n_bad = bad > 0 ? bad : 0;
+  if (bad < 0) {
+    set_error("elasto_check_guards: CUDA error while checking: " + std::string(cudaGetErrorString(cudaGetLastError())));
+    return ELASTO_ERR_CUDA;
+  }
+  if (bad > 0) {
+    set_error("elasto_check_guards: " + std::to_string(bad) + " guard zone(s) overwritten; first after " + first);
+    return ELASTO_ERR_GUARD;
+  }
+  return ELASTO_OK;
+}
+
+elasto_status elasto_debug_damage_guard(elasto_t h, int zone) {
+  if (!h) {
+    set_error("elasto_debug_damage_guard: null handle");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  char* base = h->arena;
+  GuardedArena* g = &h->guards;
+  if (h->cnn) g = cnn_guards(h->cnn, &base);
+  if (zone < 0 || zone >= static_cast<int>(g->zones.size()) || !base) {
+    set_error("elasto_debug_damage_guard: zone out of range");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  ELASTO_CUDA_TRY(cudaDeviceSynchronize());
+  ELASTO_CUDA_TRY(cudaMemset(base + g->zones[zone].off, 0x5A, 1));
+  ELASTO_CUDA_TRY(cudaDeviceSynchronize());
+  return ELASTO_OK;
+}
 
 elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value) {
   if (!h || !value) {
@@ -1094,6 +1133,7 @@ elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value) {
     case ELASTO_Q_LAUNCHES: *value = h->modes[mode].launches; break;
     case ELASTO_Q_PACKED_TOTAL: *value = int64_t(h->packed_total); break;
     case ELASTO_Q_PREFIX_SHARED: *value = h->prefix_shared ? 1 : 0; break;
+    case ELASTO_Q_GUARD_ZONES: *value = int64_t(h->guards.zones.size()); break;
     default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
   }
   return ELASTO_OK;

@@ -40,6 +40,7 @@
 
 #include "common.h"
 #include "elasto_internal.h"
+#include "guard.h"
 
 namespace elasto {
 
@@ -91,6 +92,7 @@ struct CnnModel {
   int n_modes = 0;
   Profiler prof;
   char* arena = nullptr;
+  GuardedArena guards;  // guard zone after every arena buffer
   size_t arena_bytes = 0, shared_bytes = 0, workspace_bytes = 0;
   int h1 = 0, w1 = 0, hp = 0, wp = 0;  // stem output and pooled sizes
   std::vector<BlockShape> shapes;
@@ -392,16 +394,6 @@ struct Bn {
   double bias(int o) const { return b[o] - mean[o] * scale(o); }
 };
 
-struct Arena {
-  size_t off = 0;
-  size_t take(size_t bytes) {
-    off = (off + kAlignB - 1) / kAlignB * kAlignB;
-    const size_t r = off;
-    off += bytes;
-    return r;
-  }
-};
-
 elasto_launch_record rec(int kind, int layer, int m, int n, int k, double macs, double bytes) {
   elasto_launch_record r{};
   r.kind = kind;
@@ -500,7 +492,7 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
   const int t_fc = ti;
 
   // ---------------------------------------------------------------- layout
-  Arena ar;
+  GuardedArena& ar = m->guards;  // every buffer followed by a guard zone
   const size_t o_stem_w = ar.take(size_t(kStemC) * kStemKs * 2), o_stem_b = ar.take(kStemC * 4);
   std::vector<size_t> o_dw(nblk, 0), o_db(nblk, 0);
   for (int i = 0; i < nblk; ++i)
@@ -551,12 +543,14 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
     if (b.proj) scb = std::max(scb, ro * 4 * size_t(b.w));
   }
   const size_t ws_start = ar.off;
-  const size_t o_s2d = ar.take(s2d * 2), o_xa = ar.take(xbuf * 2), o_xb = ar.take(xbuf * 2);
-  const size_t o_t1 = ar.take(t1 * 2), o_t2 = ar.take(t2 * 2), o_sc = ar.take(scb * 2);
-  const size_t o_pool = ar.take(size_t(Bm) * 2048 * 4);
-  const size_t o_img = ar.take(size_t(Bm) * d->img_h * d->img_w * 3 * (dt == ELASTO_BF16 ? 2 : 4));
-  const size_t o_logit = ar.take(size_t(Bm) * C * 4);
-  const size_t o_status = ar.take(64);
+  const size_t o_s2d = ar.take(s2d * 2, "space-to-depth image"), o_xa = ar.take(xbuf * 2, "activation A"),
+               o_xb = ar.take(xbuf * 2, "activation B");
+  const size_t o_t1 = ar.take(t1 * 2, "conv1 output"), o_t2 = ar.take(t2 * 2, "conv2 output"),
+               o_sc = ar.take(scb * 2, "projection shortcut");
+  const size_t o_pool = ar.take(size_t(Bm) * 2048 * 4, "pooled features");
+  const size_t o_img = ar.take(size_t(Bm) * d->img_h * d->img_w * 3 * (dt == ELASTO_BF16 ? 2 : 4), "image staging");
+  const size_t o_logit = ar.take(size_t(Bm) * C * 4, "logit staging");
+  const size_t o_status = ar.take(64, "status word");
   m->workspace_bytes = ar.off - ws_start;
   m->arena_bytes = ar.off;
 
@@ -569,6 +563,10 @@ elasto_status cnn_create(const elasto_model_desc* d, const elasto_weights* wts, 
   }
   char* A = m->arena;
   ELASTO_CUDA_TRY(cudaMemset(A, 0, m->arena_bytes));
+  {
+    const elasto_status gs = m->guards.upload(A);
+    if (gs != ELASTO_OK) return gs;
+  }
   m->stem_w = reinterpret_cast<F16Buf*>(A + o_stem_w);
   m->stem_b = reinterpret_cast<float*>(A + o_stem_b);
   m->down_w.assign(nblk, nullptr);
@@ -839,6 +837,7 @@ void cnn_destroy(CnnModel* m) {
     cudaDeviceSynchronize();
     cudaFree(m->arena);
   }
+  m->guards.release();
   m->prof.release();
   delete m;
 }
@@ -864,6 +863,7 @@ elasto_status cnn_query(CnnModel* m, int what, int mode, int64_t* value) {
       break;
     }
     case ELASTO_Q_PREFIX_SHARED: *value = 0; break;
+    case ELASTO_Q_GUARD_ZONES: *value = int64_t(m->guards.zones.size()); break;
     default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
   }
   return ELASTO_OK;
@@ -910,6 +910,11 @@ elasto_status cnn_export_packed(CnnModel* m, int mode, int block, int which, voi
     }
   }
   return ELASTO_OK;
+}
+
+GuardedArena* cnn_guards(CnnModel* m, char** base) {
+  *base = m->arena;
+  return &m->guards;
 }
 
 }  // namespace elasto

@@ -42,6 +42,9 @@ void cnn_destroy(CnnModel* m);  // frees the model and its device memory
 elasto_status cnn_query(CnnModel* m, int what, int mode, int64_t* value);
 elasto_status cnn_export_packed(CnnModel* m, int mode, int block, int which, void* host_dst, size_t bytes);
 
+struct GuardedArena;  // guard.h
+GuardedArena* cnn_guards(CnnModel* m, char** base);  // the CNN arena's guard zones and base
+
 cudaError_t ensure_kernel_attributes();
 elasto_status check_device();
 

@@ -5,6 +5,7 @@
 
 #include "common.h"
 #include "elasto_internal.h"
+#include "guard.h"
 
 namespace elasto {
 
@@ -63,6 +64,7 @@ struct elasto_s {
   int dev = 0;
   int n = 0, np = 0, kpe = 0;
   char* arena = nullptr;
+  elasto::GuardedArena guards;  // guard zone after every arena buffer
   size_t arena_bytes = 0, shared_bytes = 0, workspace_bytes = 0;
   // shared (mode-independent) parameters
   elasto::bf16* patch_w = nullptr;

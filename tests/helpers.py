@@ -60,6 +60,8 @@ def centred_tolerance(ref: np.ndarray, layers: int, roundings_per_layer: int = 5
     which is a share s of max|logit|, that is 2^-9 * sqrt(5 L) / s; never
     below 2e-2."""
     share = float(np.max(np.abs(centered(ref))) / np.max(np.abs(ref)))
+    if share == 0.0:  # one image: nothing varies across the batch
+        return float("inf")
     return max(2e-2, BF16_U * np.sqrt(roundings_per_layer * layers) / share)
 
 

@@ -234,7 +234,7 @@ def test_nested_modes_share_one_packed_copy(cfg):
         total = model.query(binding.Q_PACKED_TOTAL)
         views = [model.query(binding.Q_PACKED_BYTES, m) for m in range(len(tables))]
         assert views[0] == max(views)
-        assert total <= views[0] + 1024 * 6 * cfg.layers  # alignment slack only
+        assert total <= views[0] + 2048 * 10 * cfg.layers  # alignment and guard zones only (<= 2 KiB a buffer)
         assert total < sum(views)
         x = dev(img)
         for m in (0, len(tables) - 1):
