@@ -45,6 +45,8 @@ def test_null_handle_calls_fail_cleanly(lib):
     assert "null handle" in binding.elasto_last_error()
     assert lib.elasto_forward(None, None, None, 1, None) == binding.ERR_INVALID_ARG
     assert lib.elasto_destroy(None) == binding.ERR_INVALID_ARG
+    assert lib.elasto_check_guards(None, None, None) == binding.ERR_INVALID_ARG
+    assert lib.elasto_debug_damage_guard(None, 0) == binding.ERR_INVALID_ARG
     v = ctypes.c_int64()
     assert lib.elasto_query(None, 0, 0, ctypes.byref(v)) == binding.ERR_INVALID_ARG
 
