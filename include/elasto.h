@@ -158,6 +158,25 @@ elasto_status elasto_forward(elasto_t h, void* stream, const void* images_device
 elasto_status elasto_forward_host(elasto_t h, void* stream, const void* images_host, int batch,
                                   float* logits_host);
 
+/* A sequence of forwards from host memory with the copies overlapped (the
+ * serving loop of Section 4.4's runtime: one DN, batches arriving in host
+ * memory). Batch i (batch images, all batches of one size) is read from
+ * images_host[i] ([batch, img_h, img_w, img_c] NHWC of weight_dtype) and its
+ * logits are written to logits_host[i] ([batch, classes] fp32); the two
+ * pointer arrays have n_batches entries. Batch i+1's images are copied to
+ * the device on one library stream while batch i's forward runs on `stream`,
+ * and batch i's logits come back on another while batch i+1 runs, through
+ * two library-owned device staging pairs (the second is allocated by the
+ * first call on a handle, as are the two copy streams and their events).
+ * Returns when every logit is in host memory. Host buffers must be pinned
+ * (cudaHostAlloc / cudaHostRegister) for the copies to overlap; pageable
+ * memory works but serialises them. Every batch runs in the mode current at
+ * the call (as for elasto_forward, set_mode must not run concurrently).
+ * Errors: INVALID_ARG (null pointer, n_batches < 1, batch outside
+ * [1, max_batch]), OOM, CUDA. */
+elasto_status elasto_forward_host_batches(elasto_t h, void* stream, int n_batches, int batch,
+                                          const void* const* images_host, float* const* logits_host);
+
 /* The same forward as elasto_forward (ViT handles), for callers that must not
  * allocate device memory when they run inference: e.g. a process whose
  * memory manager takes the whole GPU into its own pool at start-up and

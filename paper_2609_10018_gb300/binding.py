@@ -86,6 +86,8 @@ def lib() -> ctypes.CDLL:
         "elasto_get_mode": [c_void_p, ctypes.POINTER(c_int)],
         "elasto_forward": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
         "elasto_forward_host": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
+        "elasto_forward_host_batches": [c_void_p, c_void_p, c_int, c_int, ctypes.POINTER(c_void_p),
+                                        ctypes.POINTER(c_void_p)],
         "elasto_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_int, c_void_p],
         "elasto_sync_status": [c_void_p, c_void_p],
         "elasto_check_guards": [c_void_p, c_void_p, ctypes.POINTER(c_int)],
@@ -233,6 +235,20 @@ def elasto_forward_host(h: int, stream: int, images: np.ndarray, batch: int, log
     assert images.flags["C_CONTIGUOUS"] and logits.flags["C_CONTIGUOUS"] and logits.dtype == np.float32
     _check(lib().elasto_forward_host(h, stream, images.ctypes.data, batch, logits.ctypes.data),
            "elasto_forward_host")
+
+
+def elasto_forward_host_batches(h: int, stream: int, images: List[np.ndarray], logits: List[np.ndarray]) -> None:
+    """Batches from host memory, copies overlapped with the forwards (all
+    batches the same size; pinned host arrays for the overlap)."""
+    n = len(images)
+    assert n == len(logits) and n > 0
+    for a in list(images) + list(logits):
+        assert a.flags["C_CONTIGUOUS"]
+    assert all(l.dtype == np.float32 for l in logits)
+    ip = (c_void_p * n)(*[a.ctypes.data for a in images])
+    lp = (c_void_p * n)(*[a.ctypes.data for a in logits])
+    _check(lib().elasto_forward_host_batches(h, stream, n, images[0].shape[0], ip, lp),
+           "elasto_forward_host_batches")
 
 
 def elasto_sync_status(h: int, stream: int = 0) -> None:
@@ -415,6 +431,9 @@ class ElasticModel:
 
     def forward_host(self, images: np.ndarray, logits: np.ndarray, stream: int = 0) -> None:
         elasto_forward_host(self.handle, stream, images, images.shape[0], logits)
+
+    def forward_host_batches(self, images: List[np.ndarray], logits: List[np.ndarray], stream: int = 0) -> None:
+        elasto_forward_host_batches(self.handle, stream, images, logits)
 
     def sync_status(self, stream: int = 0) -> None:
         elasto_sync_status(self.handle, stream)

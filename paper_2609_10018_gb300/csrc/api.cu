@@ -1037,6 +1037,79 @@ elasto_status elasto_forward_host(elasto_t h, void* stream, const void* images_h
   return ELASTO_OK;
 }
 
+elasto_status elasto_forward_host_batches(elasto_t h, void* stream, int n_batches, int batch,
+                                          const void* const* images_host, float* const* logits_host) {
+  if (!h || !images_host || !logits_host || n_batches < 1) {
+    set_error("elasto_forward_host_batches: null argument or n_batches < 1");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  if (batch < 1 || batch > h->d.max_batch) {
+    set_error("elasto_forward_host_batches: batch outside [1, max_batch]");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  for (int i = 0; i < n_batches; ++i)
+    if (!images_host[i] || !logits_host[i]) {
+      set_error("elasto_forward_host_batches: null buffer for batch " + std::to_string(i));
+      return ELASTO_ERR_INVALID_ARG;
+    }
+  const size_t img_cap = size_t(h->d.max_batch) * h->d.img_h * h->d.img_w * h->d.img_c * dtype_size(h->d.weight_dtype);
+  const size_t logit_cap = size_t(h->d.max_batch) * h->d.classes * 4;
+  if (!h->stage2) {  // first call: the second staging pair, streams and events
+    cudaError_t e = cudaMalloc(&h->stage2, img_cap + 256 + logit_cap);
+    if (e != cudaSuccess) {
+      h->stage2 = nullptr;
+      cudaGetLastError();
+      set_error("elasto_forward_host_batches: cudaMalloc of the second staging pair failed");
+      return ELASTO_ERR_OOM;
+    }
+    ELASTO_CUDA_TRY(cudaStreamCreateWithFlags(&h->h2d, cudaStreamNonBlocking));
+    ELASTO_CUDA_TRY(cudaStreamCreateWithFlags(&h->d2h, cudaStreamNonBlocking));
+    for (int k = 0; k < 2; ++k) {
+      ELASTO_CUDA_TRY(cudaEventCreateWithFlags(&h->ev_h2d[k], cudaEventDisableTiming));
+      ELASTO_CUDA_TRY(cudaEventCreateWithFlags(&h->ev_fwd[k], cudaEventDisableTiming));
+      ELASTO_CUDA_TRY(cudaEventCreateWithFlags(&h->ev_d2h[k], cudaEventDisableTiming));
+    }
+  }
+  void* img[2] = {h->cnn ? cnn_image_stage(h->cnn) : h->img_stage, h->stage2};
+  float* lg[2] = {h->cnn ? cnn_logit_stage(h->cnn) : h->logit_stage,
+                  reinterpret_cast<float*>(h->stage2 + (img_cap + 255) / 256 * 256)};
+  const size_t ib = size_t(batch) * h->d.img_h * h->d.img_w * h->d.img_c * dtype_size(h->d.weight_dtype);
+  const size_t lb = size_t(batch) * h->d.classes * 4;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // the copy streams start after the work already on `stream` (which may
+  // still be using the staging buffers)
+  ELASTO_CUDA_TRY(cudaEventRecord(h->ev_fwd[0], s));
+  ELASTO_CUDA_TRY(cudaEventRecord(h->ev_fwd[1], s));
+  ELASTO_CUDA_TRY(cudaEventRecord(h->ev_d2h[0], s));
+  ELASTO_CUDA_TRY(cudaEventRecord(h->ev_d2h[1], s));
+  // batch 0's images
+  ELASTO_CUDA_TRY(cudaStreamWaitEvent(h->h2d, h->ev_fwd[0], 0));
+  ELASTO_CUDA_TRY(cudaMemcpyAsync(img[0], images_host[0], ib, cudaMemcpyHostToDevice, h->h2d));
+  ELASTO_CUDA_TRY(cudaEventRecord(h->ev_h2d[0], h->h2d));
+  for (int i = 0; i < n_batches; ++i) {
+    const int cb = i & 1, nb = cb ^ 1;
+    if (i + 1 < n_batches) {
+      // batch i+1's images into the other staging buffer once the forward
+      // that last read it (batch i-1) is done
+      ELASTO_CUDA_TRY(cudaStreamWaitEvent(h->h2d, h->ev_fwd[nb], 0));
+      ELASTO_CUDA_TRY(cudaMemcpyAsync(img[nb], images_host[i + 1], ib, cudaMemcpyHostToDevice, h->h2d));
+      ELASTO_CUDA_TRY(cudaEventRecord(h->ev_h2d[nb], h->h2d));
+    }
+    // batch i: its images are in, and batch i-2's logits have left lg[cb]
+    ELASTO_CUDA_TRY(cudaStreamWaitEvent(s, h->ev_h2d[cb], 0));
+    ELASTO_CUDA_TRY(cudaStreamWaitEvent(s, h->ev_d2h[cb], 0));
+    const elasto_status st = elasto_forward(h, stream, img[cb], batch, lg[cb]);
+    if (st != ELASTO_OK) return st;
+    ELASTO_CUDA_TRY(cudaEventRecord(h->ev_fwd[cb], s));
+    ELASTO_CUDA_TRY(cudaStreamWaitEvent(h->d2h, h->ev_fwd[cb], 0));
+    ELASTO_CUDA_TRY(cudaMemcpyAsync(logits_host[i], lg[cb], lb, cudaMemcpyDeviceToHost, h->d2h));
+    ELASTO_CUDA_TRY(cudaEventRecord(h->ev_d2h[cb], h->d2h));
+  }
+  ELASTO_CUDA_TRY(cudaStreamSynchronize(h->d2h));
+  ELASTO_CUDA_TRY(cudaStreamSynchronize(s));
+  return ELASTO_OK;
+}
+
 elasto_status elasto_sync_status(elasto_t h, void* stream) {
   if (!h) {
     set_error("elasto_sync_status: null handle");
@@ -1063,6 +1136,14 @@ elasto_status elasto_destroy(elasto_t h) {
   if (h->arena) cudaFree(h->arena);
   if (h->cnn) cnn_destroy(h->cnn);
   noalloc_cache_free(h->noalloc);
+  if (h->stage2) cudaFree(h->stage2);
+  if (h->h2d) cudaStreamDestroy(h->h2d);
+  if (h->d2h) cudaStreamDestroy(h->d2h);
+  for (int k = 0; k < 2; ++k) {
+    if (h->ev_h2d[k]) cudaEventDestroy(h->ev_h2d[k]);
+    if (h->ev_fwd[k]) cudaEventDestroy(h->ev_fwd[k]);
+    if (h->ev_d2h[k]) cudaEventDestroy(h->ev_d2h[k]);
+  }
   h->guards.release();
   h->prof.release();
   delete h;

@@ -95,6 +95,11 @@ struct elasto_s {
   std::vector<std::vector<int32_t>> perm_h, perm_f;
   size_t packed_total = 0;  // device bytes of all modes' packed weights
   std::atomic<int> cur{0};
+  // elasto_forward_host_batches: a second device staging pair (images, then
+  // logits) and the copy streams / events, made by its first call
+  char* stage2 = nullptr;
+  cudaStream_t h2d = nullptr, d2h = nullptr;
+  cudaEvent_t ev_h2d[2] = {}, ev_fwd[2] = {}, ev_d2h[2] = {};
   elasto::NoallocCache* noalloc = nullptr;  // built by the first elasto_forward_noalloc call
   // CNN state lives behind this pointer (null for ViT)
   elasto::CnnModel* cnn = nullptr;

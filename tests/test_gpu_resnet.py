@@ -115,6 +115,20 @@ def test_resnet_packed_weights_match_oracle_folding():
                         assert np.allclose(got, ref, rtol=1e-6, atol=1e-7), (m, i, which)
 
 
+def test_resnet_forward_host_batches_equals_device_forward():
+    import torch
+    cfg = SMALL
+    w, tables = synth.make_resnet_weights(cfg), synth.make_resnet_tables(cfg)
+    nb, B = 4, 2
+    imgs = [torch.from_numpy(synth.make_images(cfg, B, seed=200 + i)).pin_memory().numpy() for i in range(nb)]
+    with binding.ElasticModel.resnet(cfg, w, tables, max_batch=B) as model:
+        model.set_mode(3)
+        outs = [np.zeros((B, cfg.classes), np.float32) for _ in range(nb)]
+        model.forward_host_batches(imgs, outs)
+        for i in range(nb):
+            assert np.array_equal(outs[i].astype(np.float64), _run(model, dev(imgs[i]), B, cfg.classes, 3)), i
+
+
 def test_resnet_batch_1_and_ragged_and_switch():
     cfg = SMALL
     w, tables = synth.make_resnet_weights(cfg), synth.make_resnet_tables(cfg)

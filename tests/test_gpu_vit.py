@@ -199,6 +199,28 @@ def test_forward_host_equals_device_forward(tiny):
         assert np.array_equal(host_out.astype(np.float64), dev_out)
 
 
+def test_forward_host_batches_equals_device_forward(tiny):
+    """Batches streamed from (pinned) host memory with the copies overlapped:
+    every batch's logits equal the device forward of the same images bit for
+    bit, in both modes, with batches alternating between the two staging
+    buffers."""
+    import torch
+    cfg, w, wide, tables = tiny
+    nb, B = 5, 3
+    imgs = [torch.from_numpy(synth.make_images(cfg, B, seed=100 + i)).pin_memory().numpy() for i in range(nb)]
+    with binding.ElasticModel.vit(cfg, w, tables, max_batch=4) as model:
+        for m in range(len(tables)):
+            model.set_mode(m)
+            outs = [torch.zeros((B, cfg.classes), dtype=torch.float32).pin_memory().numpy() for _ in range(nb)]
+            model.forward_host_batches(imgs, outs)
+            for i in range(nb):
+                assert np.array_equal(outs[i].astype(np.float64), _run(model, dev(imgs[i]), B, cfg.classes, m)), (m, i)
+        with pytest.raises(binding.ElastoError) as e:
+            model.forward_host_batches([np.zeros((5,) + imgs[0].shape[1:], imgs[0].dtype)],
+                                       [np.zeros((5, cfg.classes), np.float32)])
+        assert e.value.status == binding.ERR_INVALID_ARG
+
+
 def test_degenerate_and_non_nested_tables():
     """Layers keeping no head and/or no MLP channel, a channel count that is
     not a multiple of 8, and tables that are not nested across modes."""
