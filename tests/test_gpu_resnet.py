@@ -67,10 +67,10 @@ def test_resnet50_small_all_modes_2000_images():
 
 
 def test_resnet50_224_all_modes():
-    """224x224 (ImageNet-shaped), 64 images per mode."""
+    """224x224 (ImageNet-shaped), 128 images per mode (the bench's batch)."""
     cfg = synth.RESNET50
     w, tables = synth.make_resnet_weights(cfg), synth.make_resnet_tables(cfg)
-    n_img = 64
+    n_img = 128
     img = synth.make_images(cfg, n_img)
     with binding.ElasticModel.resnet(cfg, w, tables, max_batch=n_img) as model:
         x = dev(img)
