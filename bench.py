@@ -400,6 +400,8 @@ def main():
     if rank == 0 and not args.quick:
         line["embed_ladder"] = embed_ladder(torch, binding, synth, weights, images, peaks)
         line["resnet50"] = resnet50_section(torch, binding, synth, peaks)
+        line["vit_s16"] = small_vit_section(torch, binding, synth, synth.VIT_S, peaks)
+        line["tiny_vit"] = small_vit_section(torch, binding, synth, synth.TINY, peaks)
     if rank == 0:
         print(json.dumps(line))
     if dist:
@@ -458,6 +460,40 @@ def embed_ladder(torch, binding, synth, weights, images, peaks, cr=0.4, rounds=5
     model.close()
     return {"batch": B, "cr": cr, "rounds": rounds, "levels": out,
             "note": "Table 1 counts FLOPs as multiply-accumulates of the linear layers; gmac_per_image adds attention"}
+
+
+def small_vit_section(torch, binding, synth, cfg, peaks, warmup=10, trials=50):
+    """The other ViT configurations at their own batch (ViT-S/16 at 64, the
+    tiny elastic ViT at 8): every mode, 10 warm-up + 50 timed back-to-back
+    forwards, per-forward CUDA-event latency p50 / p99 and images/s."""
+    B = cfg.batch
+    w, tables = synth.make_vit_weights(cfg), synth.make_vit_tables(cfg)
+    model = binding.ElasticModel.vit(cfg, w, tables, max_batch=B)
+    img = torch.from_numpy(synth.make_images(cfg, B)).cuda()
+    lg = torch.empty(B, cfg.classes, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    out = {"workload": f"elastic {cfg.name} DN forward, {cfg.img}x{cfg.img}, batch {B}", "per_mode": []}
+    for m in range(len(tables)):
+        model.set_mode(m)
+        for _ in range(warmup):
+            model.forward(sh, img.data_ptr(), B, lg.data_ptr())
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(trials)]
+        torch.cuda.synchronize()
+        for e0, e1 in ev:
+            e0.record(stream)
+            model.forward(sh, img.data_ptr(), B, lg.data_ptr())
+            e1.record(stream)
+        torch.cuda.synchronize()
+        ts = [e0.elapsed_time(e1) for e0, e1 in ev]
+        ips = B * trials / (sum(ts) / 1e3)
+        macs = model.query(binding.Q_MODE_MACS, m)
+        out["per_mode"].append({"mode": m, "heads": int(len(tables[m]["heads"][0])),
+                                "mlp": int(len(tables[m]["mlp"][0])), "images_per_s": ips,
+                                "ms_p50": statistics.median(ts), "ms_p99": float(np.percentile(ts, 99)),
+                                "frac_of_bf16_peak": 2.0 * macs * ips / 1e12 / peaks["bf16_tflops"]})
+    model.close()
+    return out
 
 
 def resnet50_section(torch, binding, synth, peaks, B=128, steps=20, warmup=3):
