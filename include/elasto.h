@@ -240,15 +240,44 @@ enum {
   ELASTO_Q_WORKSPACE_BYTES = 3,  /* activation workspace for max_batch */
   ELASTO_Q_ARENA_BYTES = 4,      /* total device bytes owned by the handle */
   ELASTO_Q_MODE_MACS = 5,        /* multiply-accumulates per image of the mode */
-  ELASTO_Q_LAUNCHES = 6,         /* kernels one forward of the mode launches (a one-image ViT
-                                    forward launches at most one more: its out-projection and FC2 run
-                                    split-K, their partial-sum launches compute the LayerNorms
-                                    that follow, and the last FC2's sum stands alone) */
+  ELASTO_Q_LAUNCHES = 6,         /* kernels one forward of the mode launches kernel by kernel
+                                    (a one-image ViT forward launches at most one more: its
+                                    out-projection and FC2 run split-K, their partial-sum
+                                    launches compute the LayerNorms that follow, and the last
+                                    FC2's sum stands alone); a one-image forward with a
+                                    one-launch plan (ELASTO_Q_ONE_LAUNCH) launches 1 */
   ELASTO_Q_PACKED_TOTAL = 7,     /* device bytes of all modes' packed weights together */
   ELASTO_Q_PREFIX_SHARED = 8,    /* 1 if the modes share one prefix-ordered packed copy */
-  ELASTO_Q_GUARD_ZONES = 9       /* guard zones in the handle's arena (elasto_check_guards) */
+  ELASTO_Q_GUARD_ZONES = 9,      /* guard zones in the handle's arena (elasto_check_guards) */
+  ELASTO_Q_ONE_LAUNCH = 10       /* 1 if the mode's one-image forwards run as one launch
+                                    (elasto_set_one_launch), else 0 */
 };
 elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value);
+
+/* One-image forwards as one launch (ViT handles; the paper has no
+ * counterpart: Section 6.2 measures DN latency at batch 1, where a forward of
+ * ~88 dependent kernels is bound by their launch and ramp-up latencies).
+ * With it on (off by default), elasto_forward with batch == 1 runs the whole DN
+ * forward (patch rows, patch projection, every layer, final norm and
+ * classifier) as the phases of one persistent cooperative kernel with one
+ * block per SM, preceded by an 8-byte cudaMemsetAsync of its barrier words:
+ * the same operations, the same packed weights and the same handle workspace
+ * as the kernel-by-kernel forward; results agree within floating-point
+ * reassociation (the LayerNorm sums and the split-K partitions differ), not
+ * bit for bit. Plans are made at create time for every mode that fits
+ * (bf16-stored weights, at most 256 tokens, embedding width <= 1024);
+ * elasto_query(ELASTO_Q_ONE_LAUNCH, mode) says which (0 while it is off).
+ * Measured on GB300 it is slower than the kernel-by-kernel forward (ViT-B/16
+ * 0.61 against 0.51 ms): each of its ~88 phases pays a grid barrier and the
+ * latency of its first loads, as each launch of the chain does, and the chain
+ * overlaps a launch's set-up with the previous kernel (programmatic dependent
+ * launch); it is kept as an alternative, tested like the default path.
+ * Phases are separated by grid-wide barriers whose waits are bounded; a wait
+ * that gives up records ELASTO_ERR_TIMEOUT in the status word and the launch
+ * ends. Forwards of one handle must not overlap on the GPU (as for every
+ * forward: they share its workspace). No effect on ResNet-50 handles.
+ * Errors: INVALID_ARG (null handle). */
+elasto_status elasto_set_one_launch(elasto_t h, int enable);
 
 /* Per-launch timing (diagnostics). While enabled, forward records a CUDA
  * event pair around every kernel it launches; elasto_profile_read
@@ -260,7 +289,8 @@ enum {
   ELASTO_K_PATCHIFY = 0, ELASTO_K_GEMM = 1, ELASTO_K_LAYERNORM = 2, ELASTO_K_ATTENTION = 3,
   ELASTO_K_HEAD = 4,
   ELASTO_K_IM2COL = 5, /* the CNN stem's input rearrangement (space-to-depth) */
-  ELASTO_K_POOL = 6
+  ELASTO_K_POOL = 6,
+  ELASTO_K_ONE_LAUNCH = 7 /* a whole one-image ViT forward in one launch (elasto_set_one_launch) */
 };
 typedef struct {
   int kind;     /* ELASTO_K_* */

@@ -23,7 +23,7 @@ F32, BF16 = 0, 1
 OK, ERR_INVALID_ARG, ERR_BAD_TABLE, ERR_BAD_MODE, ERR_OOM, ERR_CUDA, ERR_UNSUPPORTED, ERR_TIMEOUT, ERR_GUARD = (
     0, -1, -2, -3, -4, -5, -6, -7, -8)
 Q_N_MODES, Q_PACKED_BYTES, Q_SHARED_BYTES, Q_WORKSPACE_BYTES, Q_ARENA_BYTES, Q_MODE_MACS, Q_LAUNCHES = range(7)
-Q_PACKED_TOTAL, Q_PREFIX_SHARED, Q_GUARD_ZONES = 7, 8, 9
+Q_PACKED_TOTAL, Q_PREFIX_SHARED, Q_GUARD_ZONES, Q_ONE_LAUNCH = 7, 8, 9, 10
 EPI_BIAS_BF16, EPI_BIAS_GELU_BF16, EPI_BIAS_RESID_F32, EPI_BIAS_F32, EPI_BIAS_RELU_BF16, EPI_BIAS_RESID_RELU_BF16 = range(6)
 EPI_BIAS_RELU_F16, EPI_BIAS_F16, EPI_BIAS_RESID_RELU_F16 = range(6, 9)  # A, W, resid, out in IEEE f16
 
@@ -47,9 +47,9 @@ class ModeTables(ctypes.Structure):
                 ("embed_kept", P_i32), ("n_embed_kept", ctypes.c_int32)]
 
 
-K_PATCHIFY, K_GEMM, K_LAYERNORM, K_ATTENTION, K_HEAD, K_IM2COL, K_POOL = range(7)
+K_PATCHIFY, K_GEMM, K_LAYERNORM, K_ATTENTION, K_HEAD, K_IM2COL, K_POOL, K_ONE_LAUNCH = range(8)
 KIND_NAMES = {K_PATCHIFY: "patchify", K_GEMM: "gemm", K_LAYERNORM: "layernorm", K_ATTENTION: "attention",
-              K_HEAD: "head", K_IM2COL: "im2col", K_POOL: "pool"}
+              K_HEAD: "head", K_IM2COL: "im2col", K_POOL: "pool", K_ONE_LAUNCH: "one_launch"}
 
 
 class DnProfile(ctypes.Structure):
@@ -96,6 +96,7 @@ def lib() -> ctypes.CDLL:
         "elasto_query": [c_void_p, c_int, c_int, ctypes.POINTER(c_int64)],
         "elasto_debug_export_packed": [c_void_p, c_int, c_int, c_int, c_void_p, c_size_t],
         "elasto_profile_enable": [c_void_p, c_int],
+        "elasto_set_one_launch": [c_void_p, c_int],
         "elasto_profile_read": [c_void_p, ctypes.POINTER(LaunchRecord), c_int, ctypes.POINTER(c_int)],
         "elasto_profile_dns": [c_void_p, c_void_p, c_int, c_int, ctypes.POINTER(DnProfile)],
         "elasto_select_dn": [ctypes.POINTER(DnProfile), c_int, ctypes.c_float, ctypes.c_double, ctypes.c_float,
@@ -283,6 +284,10 @@ def elasto_debug_export_packed(h: int, mode: int, layer: int, which: int, out: n
     return out
 
 
+def elasto_set_one_launch(h: int, enable: bool) -> None:
+    _check(lib().elasto_set_one_launch(h, 1 if enable else 0), "elasto_set_one_launch")
+
+
 def elasto_profile_enable(h: int, enable: bool) -> None:
     _check(lib().elasto_profile_enable(h, 1 if enable else 0), "elasto_profile_enable")
 
@@ -448,6 +453,10 @@ class ElasticModel:
 
     def profile(self, enable: bool) -> None:
         elasto_profile_enable(self.handle, enable)
+
+    def set_one_launch(self, enable: bool) -> None:
+        """One-image forwards as one persistent launch, or kernel by kernel (the default)."""
+        elasto_set_one_launch(self.handle, enable)
 
     def profile_read(self) -> List[dict]:
         return elasto_profile_read(self.handle)

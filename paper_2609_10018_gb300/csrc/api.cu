@@ -55,6 +55,7 @@ cudaError_t ensure_kernel_attributes() {
     cudaError_t r = gemm_init_attributes();
     if (r == cudaSuccess) r = attn_init_attributes();
     if (r == cudaSuccess) r = cnn_init_attributes();
+    if (r == cudaSuccess) r = pk_init_attributes();
     g_attr_err[dev] = r;
   });
   return g_attr_err[dev];
@@ -403,6 +404,8 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   const size_t img_bytes = size_t(Bm) * d->img_h * d->img_w * d->img_c * dtype_size(d->weight_dtype);
   const size_t o_img = bump.take(img_bytes, "image staging"), o_logit = bump.take(size_t(Bm) * C * 4, "logit staging");
   const size_t o_status = bump.take(64, "status word");
+  const size_t o_pk_sync = bump.take(64, "one-launch barrier words");
+  const size_t o_pk_y32 = bump.take(pk_workspace_floats(D) * 4, "one-launch class-token row");
   h->workspace_bytes = bump.off - ws_start;
   h->arena_bytes = bump.off;
 
@@ -442,6 +445,8 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
   h->img_stage = A + o_img;
   h->logit_stage = reinterpret_cast<float*>(A + o_logit);
   h->status = reinterpret_cast<int*>(A + o_status);
+  h->pk_sync = reinterpret_cast<unsigned*>(A + o_pk_sync);
+  h->pk_y32 = reinterpret_cast<float*>(A + o_pk_y32);
   for (int m = 0; m < n_modes; ++m) {
     VitEmbed& em = h->modes[m].emb;
     if (!em.pruned) {  // the handle's full-width parameters
@@ -859,7 +864,8 @@ elasto_status vit_create(const elasto_model_desc* d, const elasto_weights* wts, 
       vm.launches += 2;
     }
   }
-  return ELASTO_OK;
+  // one-image forwards as one persistent launch, where the mode allows it
+  return pk_build(h, h->pk_sync, h->pk_y32, &h->pk);
 }
 
 elasto_launch_record make_rec(int kind, int layer, int m, int n, int k, double macs, double bytes) {
@@ -891,12 +897,22 @@ elasto_launch_record gemm_rec(int layer, int M, int N, int K, int out_bytes, boo
 
 elasto_status vit_forward(elasto_s* h, cudaStream_t s, const void* images, int batch, float* logits) {
   const elasto_model_desc& d = h->d;
-  const VitMode& vm = h->modes[h->cur.load(std::memory_order_acquire)];
+  const int mode = h->cur.load(std::memory_order_acquire);
+  const VitMode& vm = h->modes[mode];
   const int n = h->n, D = d.dim, M = batch * n, Mp = batch * h->np, C = d.classes;
   const double img_elt = d.weight_dtype == ELASTO_BF16 ? 2 : 4;
   const VitEmbed& em = vm.emb;
   const int Dm = em.d_pad;  // residual-stream width (kept embedding channels, zero-padded)
   h->prof.begin();
+  if (batch == 1 && pk_ready(h->pk, mode)) {
+    // the whole forward as one persistent launch (csrc/persistent.cu);
+    // algorithmic bytes: the mode's weights, the image and the logits
+    ELASTO_LAUNCH(make_rec(ELASTO_K_ONE_LAUNCH, -1, n, Dm, 0, double(vm.macs),
+                           double(vm.packed_bytes + h->shared_bytes) + double(h->np) * h->kpe * img_elt +
+                               double(C) * 4),
+                  pk_launch(h->pk, mode, n, images, logits, h->status, s));
+    return ELASTO_OK;
+  }
   ELASTO_LAUNCH(make_rec(ELASTO_K_PATCHIFY, -1, M, h->kpe, 0, 0, double(Mp) * h->kpe * img_elt + double(M) * h->kpe * 2),
                 patch_rows_launch(images, d.weight_dtype, batch, d.img_h, d.img_w, d.img_c, d.patch, h->P, s));
   // patch projection; the addend (class token / position embedding / b_pe)
@@ -970,6 +986,7 @@ elasto_status elasto_create(const elasto_model_desc* desc, const elasto_weights*
     cudaDeviceSynchronize();
     if (h->arena) cudaFree(h->arena);
     h->guards.release();
+    pk_free(h->pk);
     if (h->cnn) cnn_destroy(h->cnn);
     return st;
   }
@@ -1136,6 +1153,7 @@ elasto_status elasto_destroy(elasto_t h) {
   if (h->arena) cudaFree(h->arena);
   if (h->cnn) cnn_destroy(h->cnn);
   noalloc_cache_free(h->noalloc);
+  pk_free(h->pk);
   if (h->stage2) cudaFree(h->stage2);
   if (h->h2d) cudaStreamDestroy(h->h2d);
   if (h->d2h) cudaStreamDestroy(h->d2h);
@@ -1199,7 +1217,8 @@ elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value) {
   }
   if (h->cnn) return cnn_query(h->cnn, what, mode, value);
   const int nm = static_cast<int>(h->modes.size());
-  const bool needs_mode = what == ELASTO_Q_PACKED_BYTES || what == ELASTO_Q_MODE_MACS || what == ELASTO_Q_LAUNCHES;
+  const bool needs_mode = what == ELASTO_Q_PACKED_BYTES || what == ELASTO_Q_MODE_MACS || what == ELASTO_Q_LAUNCHES ||
+                          what == ELASTO_Q_ONE_LAUNCH;
   if (needs_mode && (mode < 0 || mode >= nm)) {
     set_error("elasto_query: bad mode");
     return ELASTO_ERR_BAD_MODE;
@@ -1215,8 +1234,18 @@ elasto_status elasto_query(elasto_t h, int what, int mode, int64_t* value) {
     case ELASTO_Q_PACKED_TOTAL: *value = int64_t(h->packed_total); break;
     case ELASTO_Q_PREFIX_SHARED: *value = h->prefix_shared ? 1 : 0; break;
     case ELASTO_Q_GUARD_ZONES: *value = int64_t(h->guards.zones.size()); break;
+    case ELASTO_Q_ONE_LAUNCH: *value = pk_ready(h->pk, mode) ? 1 : 0; break;
     default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
   }
+  return ELASTO_OK;
+}
+
+elasto_status elasto_set_one_launch(elasto_t h, int enable) {
+  if (!h) {
+    set_error("elasto_set_one_launch: null handle");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  pk_enable(h->pk, enable != 0);  // ResNet-50 handles have no plan: nothing changes
   return ELASTO_OK;
 }
 

@@ -864,6 +864,7 @@ elasto_status cnn_query(CnnModel* m, int what, int mode, int64_t* value) {
     }
     case ELASTO_Q_PREFIX_SHARED: *value = 0; break;
     case ELASTO_Q_GUARD_ZONES: *value = int64_t(m->guards.zones.size()); break;
+    case ELASTO_Q_ONE_LAUNCH: *value = 0; break;  // the one-launch forward is ViT-only
     default: set_error("elasto_query: unknown query"); return ELASTO_ERR_INVALID_ARG;
   }
   return ELASTO_OK;

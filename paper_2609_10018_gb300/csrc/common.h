@@ -71,6 +71,11 @@ bool encode_tmap_4d(CUtensorMap* tm, const void* base, const uint64_t dims[4], c
 // 16-bit f16 2-D map with the 32-byte swizzle.
 bool encode_tmap_2d_sw32(CUtensorMap* tm, const void* base, uint64_t inner, uint64_t outer, uint64_t row_stride_bytes,
                          uint32_t box_inner, uint32_t box_outer);
+// Map of rank 1-5 (fp32 or bf16) for TMA stores of dense boxes: dims
+// innermost first, byte strides of dims 1..rank-1, box in elements;
+// unswizzled, or with the 128-byte swizzle (box rows of exactly 128 bytes).
+bool encode_tmap_plain(CUtensorMap* tm, const void* base, int rank, const uint64_t* dims,
+                       const uint64_t* strides_bytes, const uint32_t* box, bool fp32, bool sw128 = false);
 // 3-D bf16 tensor [d2][d1][d0] with byte strides s1 (between d1 rows) and s2.
 bool encode_tmap_3d(CUtensorMap* tm, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t s1,
                     uint64_t s2, uint32_t b0, uint32_t b1, uint32_t b2);

@@ -49,6 +49,11 @@ struct VitEmbed {
 struct NoallocCache;
 void noalloc_cache_free(NoallocCache* c);
 
+// One-launch plans of the one-image forward (csrc/persistent.cu), one per
+// mode; device memory of their own.
+struct PkPlan;
+void pk_free(PkPlan* p);
+
 struct VitMode {
   std::vector<VitLayerPack> layers;
   VitEmbed emb;
@@ -101,7 +106,25 @@ struct elasto_s {
   cudaStream_t h2d = nullptr, d2h = nullptr;
   cudaEvent_t ev_h2d[2] = {}, ev_fwd[2] = {}, ev_d2h[2] = {};
   elasto::NoallocCache* noalloc = nullptr;  // built by the first elasto_forward_noalloc call
+  elasto::PkPlan* pk = nullptr;             // one-launch plans of the one-image forward (null: none)
+  unsigned* pk_sync = nullptr;              // their grid-barrier counter and abort flag
+  float* pk_y32 = nullptr;                  // their final-norm class-token row [d]
   // CNN state lives behind this pointer (null for ViT)
   elasto::CnnModel* cnn = nullptr;
   elasto::Profiler prof;
 };
+
+namespace elasto {
+
+// csrc/persistent.cu. pk_build makes every mode's plan it can (a mode without
+// one keeps the kernel-by-kernel forward) and leaves *out null when the
+// device cannot run cooperative launches of the kernel.
+cudaError_t pk_init_attributes();
+size_t pk_workspace_floats(int d);  // floats of the class-token row buffer for width d
+elasto_status pk_build(elasto_s* h, unsigned* sync, float* y32, PkPlan** out);
+bool pk_ready(const PkPlan* p, int mode);
+void pk_enable(PkPlan* p, bool on);
+cudaError_t pk_launch(const PkPlan* p, int mode, int n, const void* images, float* logits, int* status,
+                      cudaStream_t s);
+
+}  // namespace elasto

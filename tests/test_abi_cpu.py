@@ -47,6 +47,7 @@ def test_null_handle_calls_fail_cleanly(lib):
     assert lib.elasto_destroy(None) == binding.ERR_INVALID_ARG
     assert lib.elasto_check_guards(None, None, None) == binding.ERR_INVALID_ARG
     assert lib.elasto_debug_damage_guard(None, 0) == binding.ERR_INVALID_ARG
+    assert lib.elasto_set_one_launch(None, 1) == binding.ERR_INVALID_ARG
     v = ctypes.c_int64()
     assert lib.elasto_query(None, 0, 0, ctypes.byref(v)) == binding.ERR_INVALID_ARG
 

@@ -1,7 +1,8 @@
-"""The FC1 epilogue's GELU (csrc/gemm.cu) against the exact x * Phi(x) of the
-oracle, on the CPU: the three constants are read from the kernel source and
-the same formula is evaluated in fp64, so a wrong sign, a dropped term or a
-mistyped digit in the kernel shows up here without a GPU."""
+"""The FC1 epilogue's GELU (csrc/act.cuh, used by csrc/gemm.cu and
+csrc/persistent.cu) against the exact x * Phi(x) of the oracle, on the CPU:
+the three constants are read from the kernel source and the same formula is
+evaluated in fp64, so a wrong sign, a dropped term or a mistyped digit in the
+kernel shows up here without a GPU."""
 import math
 import pathlib
 import re
@@ -11,7 +12,7 @@ import numpy as np
 from oracle import vit as ov
 from paper_2609_10018_gb300 import gelu_fit
 
-SRC = pathlib.Path(__file__).resolve().parents[1] / "paper_2609_10018_gb300" / "csrc" / "gemm.cu"
+SRC = pathlib.Path(__file__).resolve().parents[1] / "paper_2609_10018_gb300" / "csrc" / "act.cuh"
 
 
 def _kernel_constants():
