@@ -84,6 +84,17 @@ elasto_status elasto_op_attention(void* stream, const void* qkv, void* out, int 
 elasto_status elasto_op_bounded_wait(void* stream, int armed, int* status_device,
                                      unsigned long long* elapsed_ns_device);
 
+/* Self-test of the grid-wide barrier of the one-image one-launch forward
+ * (elasto_set_one_launch): a cooperative launch of one block per SM passes
+ * two barriers (arrival counter and abort flag in sync_device, 2 uint32 of
+ * device scratch, zeroed here on the stream). unreachable != 0: the second
+ * barrier waits for arrivals that never come, gives up after its limit (1 s),
+ * writes ELASTO_ERR_TIMEOUT to *status_device (if it still holds 0) and
+ * raises the abort flag, so every block returns; the context stays usable.
+ * *elapsed_ns_device (uint64): block 0's time in the two barriers. */
+elasto_status elasto_op_grid_barrier(void* stream, int unreachable, unsigned* sync_device, int* status_device,
+                                     unsigned long long* elapsed_ns_device);
+
 #ifdef __cplusplus
 }
 #endif

@@ -112,6 +112,7 @@ def lib() -> ctypes.CDLL:
         "elasto_op_softmax": [c_void_p, c_void_p, c_void_p, c_int, c_int],
         "elasto_op_attention": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p],
         "elasto_op_bounded_wait": [c_void_p, c_int, c_void_p, c_void_p],
+        "elasto_op_grid_barrier": [c_void_p, c_int, c_void_p, c_void_p, c_void_p],
     }
     for name, args in sig.items():
         f = getattr(L, name)
@@ -393,6 +394,11 @@ def elasto_op_attention(stream, qkv, out, batch, n, heads, status=0) -> None:
 
 def elasto_op_bounded_wait(stream, armed: bool, status, elapsed_ns) -> None:
     _check(lib().elasto_op_bounded_wait(stream, 1 if armed else 0, status, elapsed_ns), "elasto_op_bounded_wait")
+
+
+def elasto_op_grid_barrier(stream, unreachable: bool, sync, status, elapsed_ns) -> None:
+    _check(lib().elasto_op_grid_barrier(stream, 1 if unreachable else 0, sync, status, elapsed_ns),
+           "elasto_op_grid_barrier")
 
 
 # ----------------------------------------------------------------------------

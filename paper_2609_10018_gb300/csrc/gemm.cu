@@ -254,8 +254,14 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  pdl_wait();  // everything above overlapped the previous kernel's tail
-  pdl_trigger();
+  // Everything above overlapped the previous kernel's tail. Every thread
+  // waits for that kernel (pdl_wait) before its first access to data it may
+  // write; the weights are not such data, so the producer thread starts
+  // loading them first and waits after that.
+  if (!(warp == 0 && lane == 0 && nk > 0)) {
+    pdl_wait();
+    pdl_trigger();
+  }
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -272,6 +278,23 @@ __global__ void __launch_bounds__(THREADS, 1)
         mbar_expect_tx(bfull, static_cast<uint32_t>(nk) * bn * bke * 2);
         for (int kb = 0; kb < nk; ++kb) tma_load_2d(sB + kb * BSTG, &tmB, bfull, kb * bke, 0);
       }
+      // the first tile's first S stages: armed and their weights requested
+      // before the wait (fresh stages: no empty-slot wait needed)
+      int pre = 0;
+      if (!PAIR && !bres && t_start < tiles) {
+        const int tq = kSplit ? t_start % mn_tiles : t_start;
+        const int kb0 = kSplit ? (t_start / mn_tiles) * nk / ks : 0;
+        const int kb1 = kSplit ? (t_start / mn_tiles + 1) * nk / ks : nk;
+        const int n0 = (tq % nt) * bn;
+        pre = kb1 - kb0 < S ? kb1 - kb0 : S;
+        for (int i = 0; i < pre; ++i) {
+          mbar_expect_tx(&full[i], bytes);
+          tma_load_2d(sB + i * BSTG, &tmB, &full[i], (kb0 + i) * bke, n0);
+          if constexpr (NB == 2) tma_load_2d(sB + i * BSTG + BSTG / 2, &tmB2, &full[i], (kb0 + i) * BK, n0);
+        }
+      }
+      pdl_wait();
+      pdl_trigger();
       for (int t = t_start; t < tiles && ok; t += t_stride) {
         const int tq = kSplit ? t % mn_tiles : t;
         const int kb0 = kSplit ? (t / mn_tiles) * nk / ks : 0, kb1 = kSplit ? (t / mn_tiles + 1) * nk / ks : nk;
@@ -295,7 +318,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             continue;
           }
-          mbar_expect_tx(&full[stage], bytes);
+          const bool armed = issued < pre;  // this stage's weights were requested before the wait
+          if (!armed) mbar_expect_tx(&full[stage], bytes);
           if (args.conv) {
             const int tap = kb / args.cv_cgroups, cg = kb - tap * args.cv_cgroups;
             const int ky = tap / args.cv_ks, kx = tap - ky * args.cv_ks;
@@ -304,8 +328,9 @@ __global__ void __launch_bounds__(THREADS, 1)
           } else {
             tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
           }
-          if (!bres) tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * bke, n0);
-          if constexpr (NB == 2) tma_load_2d(sB + stage * BSTG + BSTG / 2, &tmB2, &full[stage], kb * BK, n0);
+          if (!bres && !armed) tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * bke, n0);
+          if constexpr (NB == 2)
+            if (!armed) tma_load_2d(sB + stage * BSTG + BSTG / 2, &tmB2, &full[stage], kb * BK, n0);
           ++issued;
           if (++stage == S) {
             stage = 0;

@@ -126,5 +126,8 @@ bool pk_ready(const PkPlan* p, int mode);
 void pk_enable(PkPlan* p, bool on);
 cudaError_t pk_launch(const PkPlan* p, int mode, int n, const void* images, float* logits, int* status,
                       cudaStream_t s);
+// Self-test of the one-launch forward's grid barrier (elasto_op_grid_barrier).
+cudaError_t pk_barrier_selftest(cudaStream_t s, int unreachable, unsigned* sync, int* status,
+                                unsigned long long* elapsed_ns);
 
 }  // namespace elasto

@@ -2,6 +2,7 @@
 // its own, so every kernel can be checked against the fp64 definition of that
 // step at arbitrary (odd, ragged) shapes.
 #include "common.h"
+#include "handle.h"
 #include "elasto_internal.h"
 #include "ptx.cuh"
 
@@ -44,6 +45,20 @@ elasto_status elasto_op_bounded_wait(void* stream, int armed, int* status_device
   return ELASTO_OK;
 }
 
+
+elasto_status elasto_op_grid_barrier(void* stream, int unreachable, unsigned* sync_device, int* status_device,
+                                     unsigned long long* elapsed_ns_device) {
+  clear_error();
+  if (!sync_device || !status_device || !elapsed_ns_device) {
+    set_error("elasto_op_grid_barrier: null argument");
+    return ELASTO_ERR_INVALID_ARG;
+  }
+  elasto_status st = check_device();
+  if (st != ELASTO_OK) return st;
+  ELASTO_CUDA_TRY(pk_barrier_selftest(static_cast<cudaStream_t>(stream), unreachable, sync_device, status_device,
+                                      elapsed_ns_device));
+  return ELASTO_OK;
+}
 
 elasto_status elasto_op_gemm(void* stream, const void* A, const void* W, const float* bias, void* out,
                              const void* resid, int M, int N, int K, int epilogue, int* status_device) {

@@ -759,6 +759,40 @@ __global__ void __launch_bounds__(PK_THREADS, 1)
 
 }  // namespace
 
+// ---------------------------------------------------------------- barrier self-test
+namespace {
+
+// Two grid barriers over one CTA per SM (cooperative launch, 96 threads so
+// that the polling thread 64 exists); unreachable != 0 makes the second one
+// wait for arrivals that never come, so it gives up after its limit.
+__global__ void __launch_bounds__(96) barrier_selftest_kernel(unsigned* sync, int unreachable, int* status,
+                                                                unsigned long long* elapsed_ns) {
+  __shared__ int s_ok, s_fail;
+  if (threadIdx.x == 0) s_fail = 0;
+  __syncthreads();
+  const uint64_t t0 = global_timer_ns();
+  if (grid_sync(sync, 0, status, &s_ok, &s_fail)) grid_sync(sync, unreachable ? 4 : 1, status, &s_ok, &s_fail);
+  if (blockIdx.x == 0 && threadIdx.x == 0) *elapsed_ns = global_timer_ns() - t0;
+}
+
+}  // namespace
+
+cudaError_t pk_barrier_selftest(cudaStream_t s, int unreachable, unsigned* sync, int* status,
+                                unsigned long long* elapsed_ns) {
+  cudaError_t e = cudaMemsetAsync(sync, 0, 2 * sizeof(unsigned), s);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = dim3(num_sms());
+  cfg.blockDim = dim3(96);
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeCooperative;
+  at[0].val.cooperative = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, barrier_selftest_kernel, sync, unreachable, status, elapsed_ns);
+}
+
 // ---------------------------------------------------------------- host side
 struct PkPlan {
   struct Mode {

@@ -287,3 +287,28 @@ def test_bounded_wait_gives_up_and_leaves_the_context_usable():
     assert 0.9e9 <= int(el.item()) <= 3e9 and wall < 10.0
     # the context is still usable: an attention launch right after matches the oracle
     test_attention_matches_fp64(2, 65, 2)
+
+
+def test_grid_barrier_gives_up_and_leaves_the_context_usable():
+    """The grid-wide barrier of the one-launch forward: two barriers over one
+    block per SM pass at once; a barrier waiting for arrivals that never come
+    ends after its limit with ELASTO_ERR_TIMEOUT (every block leaves through
+    the abort flag, no hang), and the context stays usable."""
+    import time
+    import torch
+    st = _status()
+    el = torch.zeros(1, dtype=torch.int64, device="cuda")
+    sync = torch.zeros(2, dtype=torch.int32, device="cuda")
+    binding.elasto_op_grid_barrier(stream_handle(), False, sync.data_ptr(), st.data_ptr(), el.data_ptr())
+    torch.cuda.synchronize()
+    assert int(st.item()) == 0
+    assert int(el.item()) < 10_000_000
+    assert int(sync[0].item()) == 2 * torch.cuda.get_device_properties(0).multi_processor_count
+    t0 = time.perf_counter()
+    binding.elasto_op_grid_barrier(stream_handle(), True, sync.data_ptr(), st.data_ptr(), el.data_ptr())
+    torch.cuda.synchronize()
+    wall = time.perf_counter() - t0
+    assert int(st.item()) == binding.ERR_TIMEOUT
+    assert int(sync[1].item()) == 1  # the abort flag
+    assert 0.9e9 <= int(el.item()) <= 3e9 and wall < 10.0
+    test_attention_matches_fp64(2, 65, 2)
