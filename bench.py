@@ -383,6 +383,15 @@ def main():
                            "note": "nested kept sets (Eq. 8): one prefix-ordered packed copy serves every mode"}
         line["batch32"] = batch32_per_mode(model, cfg, tables, torch, binding, peaks)
         line["latency"] = batch1_latency(model, cfg, tables, torch, binding, peaks)
+        if model.query(binding.Q_ONE_LAUNCH, 0) == 0:  # measure the opt-in one-launch forward beside it
+            model.set_one_launch(True)
+            if model.query(binding.Q_ONE_LAUNCH, 0) == 1:
+                line["latency_one_launch"] = {
+                    "per_mode": [{"mode": r["mode"], "us_p50": r["us_p50"], "us_p99": r["us_p99"]}
+                                 for r in batch1_latency(model, cfg, tables, torch, binding, peaks)],
+                    "note": "elasto_set_one_launch(1): the whole one-image forward as one persistent kernel "
+                            "(opt-in; the 'latency' section above is the default kernel-by-kernel forward)"}
+            model.set_one_launch(False)
         line["mode_switch_us"] = mode_switch(model, cfg, tables, torch, binding)
         lut = model.profile_dns(torch.cuda.current_stream().cuda_stream, batch=1, trials=50)
         nan = float("nan")
