@@ -227,6 +227,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     mbar_init(drain, 1);
     for (int e = 0; e < MAX_CBUFS; ++e) mbar_init(&rfull[e], 1);
     mbar_init(bfull, 1);
+    tmem_slot[1] = 0;  // the epilogue's fail flag
     fence_barrier_init();
   }
   if (warp == 0) {
@@ -443,10 +444,12 @@ __global__ void __launch_bounds__(THREADS, 1)
     const bool elected = threadIdx.x == 64;
     const int cpt = bn / CW;
     const uint32_t row_tm = tmem_base + (static_cast<uint32_t>(q * 32) << 16);
-    // One thread takes every wait decision and shares it through `verdict`,
-    // so the 128 epilogue threads always agree on whether to continue and
-    // the named barriers below can never be left one arrival short.
-    volatile int* verdict = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    // Every epilogue thread waits on the accumulator and residual barriers
+    // itself (no barrier round just to share one thread's wait); a wait that
+    // gives up raises `fail`. The flag is read only right after the chunk's
+    // named barrier, where all threads see the same value, so the 512
+    // threads leave together and the barrier is never left one arrival short.
+    volatile int* fail = reinterpret_cast<volatile int*>(tmem_slot + 1);
     ChunkIter pf;  // residual prefetch iterator (elected thread only)
     pf.init(tiles, t_start, t_stride);
     long loads = 0, consumed = 0, stored = 0;
@@ -468,13 +471,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     for (int t = t_start; t < tiles && ok; t += t_stride, ++local) {
       const int acc = local & 1;
       const uint32_t use = static_cast<uint32_t>(local >> 1);
-      if (elected)
-        *verdict = (PAIR ? mbar_wait_cluster(&tfull[acc], use & 1) : mbar_wait(&tfull[acc], use & 1)) ? 1 : 0;
-      named_bar_sync(1, EPI_THREADS);
-      if (!*verdict) {
-        ok = false;
-        break;
-      }
+      if (!(PAIR ? mbar_wait_cluster(&tfull[acc], use & 1) : mbar_wait(&tfull[acc], use & 1))) *fail = 1;
       tc_fence_after();
       const int m0 = m_tile(args, t / nt, mt) * TM + rank * BM, n0 = (t % nt) * bn;
       const uint32_t acc_tm = row_tm + acc * MAX_BN;
@@ -484,12 +481,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         uint8_t* buf = sC + e * CBUF;
         uint8_t* rowp = buf + r * 128;
         if constexpr (TR::resid) {
-          if (elected) *verdict = mbar_wait(&rfull[e], rph) ? 1 : 0;
-          named_bar_sync(1, EPI_THREADS);
-          if (!*verdict) {
-            ok = false;
-            break;
-          }
+          if (!mbar_wait(&rfull[e], rph)) *fail = 1;
           ++consumed;
         }
         {
@@ -570,6 +562,10 @@ __global__ void __launch_bounds__(THREADS, 1)
         // is written by the next chunk (E = 2) or refilled by the prefetch.
         if (elected) bulk_wait_read_all();
         named_bar_sync(1, EPI_THREADS);
+        if (*fail) {
+          ok = false;
+          break;
+        }
         if (elected) {
           if (args.conv) {
             int cb0, cy0, cx0;
