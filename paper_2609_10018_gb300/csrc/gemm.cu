@@ -50,6 +50,7 @@ namespace {
 constexpr int BM = 128, BK = 64, MAX_STAGES = 8, MAX_BN = 256;
 constexpr int EPI_THREADS = 512;                 // 16 epilogue warps, four per TMEM lane quarter
 constexpr int THREADS = 64 + EPI_THREADS;
+constexpr int THREADS_CONV = THREADS + 32;  // implicit convolutions: warp 18 is a second TMA producer
 constexpr int A_STAGE = BM * BK * 2;        // 16 KB
 constexpr int CBUF = BM * 128;              // 16 KB staging chunk (128 rows x 128 B)
 constexpr int POOL = 224 * 1024;            // operand ring + staging buffers
@@ -172,7 +173,7 @@ struct ChunkIter {
 // signals both CTAs' barriers with multicast commits; each CTA's epilogue
 // reads its own half of the accumulator from its own TMEM.
 template <int EPI, int NB, bool PAIR>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(THREADS_CONV, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const __grid_constant__ CUtensorMap tmB2,
                    const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmR,
@@ -264,23 +265,31 @@ __global__ void __launch_bounds__(THREADS, 1)
     pdl_trigger();
   }
 
-  if (warp == 0) {
+  // Implicit convolutions run two producer threads (warp 0 and warp 18,
+  // lane 0 of each) that take alternate k-blocks: issuing one 4-D box load
+  // occupies its warp for ~0.26 us, longer than the tensor core spends on a
+  // narrow k-block.
+  const int nprod = (!PAIR && args.conv && static_cast<int>(blockDim.x) == THREADS_CONV) ? 2 : 1;
+  if (warp == 0 || warp == THREADS / 32) {
     // ------------------------------------------------------------ producer
-    if (lane == 0 && nk > 0) {
+    const int pid = warp == 0 ? 0 : 1;
+    if (lane == 0 && pid < nprod && nk > 0) {
       int stage = 0;
       uint32_t phase = 0;
-      long issued = 0;
+      long seq = 0;         // k-block sequence index over this CTA's tiles
+      long last_mine = -1;  // the last k-block this thread issued
       bool ok = true;
       // pair: the even CTA's full barrier counts both CTAs' bytes
       const uint32_t bytes = PAIR ? 2 * (A_STAGE + (bn / 2) * BK * 2)
                                   : (args.conv ? args.cv_a_bytes : A_STAGE) + (bres ? 0 : NB * bn * bke * 2);
-      const bool b_loaded = bres && t_start < tiles;
+      const bool b_loaded = bres && t_start < tiles && pid == 0;
       if (b_loaded) {  // all of W, once: nk k-blocks of the single N tile
         mbar_expect_tx(bfull, static_cast<uint32_t>(nk) * bn * bke * 2);
         for (int kb = 0; kb < nk; ++kb) tma_load_2d(sB + kb * BSTG, &tmB, bfull, kb * bke, 0);
       }
       // the first tile's first S stages: armed and their weights requested
-      // before the wait (fresh stages: no empty-slot wait needed)
+      // before the wait (fresh stages: no empty-slot wait needed); thread 0
+      // issues these k-blocks
       int pre = 0;
       if (!PAIR && !bres && t_start < tiles) {
         const int tq = kSplit ? t_start % mn_tiles : t_start;
@@ -288,12 +297,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int kb1 = kSplit ? (t_start / mn_tiles + 1) * nk / ks : nk;
         const int n0 = (tq % nt) * bn;
         pre = kb1 - kb0 < S ? kb1 - kb0 : S;
-        for (int i = 0; i < pre; ++i) {
-          mbar_expect_tx(&full[i], bytes);
-          tma_load_2d(sB + i * BSTG, &tmB, &full[i], (kb0 + i) * bke, n0);
-          if constexpr (NB == 2) tma_load_2d(sB + i * BSTG + BSTG / 2, &tmB2, &full[i], (kb0 + i) * BK, n0);
-        }
+        if (pid == 0)
+          for (int i = 0; i < pre; ++i) {
+            mbar_expect_tx(&full[i], bytes);
+            tma_load_2d(sB + i * BSTG, &tmB, &full[i], (kb0 + i) * bke, n0);
+            if constexpr (NB == 2) tma_load_2d(sB + i * BSTG + BSTG / 2, &tmB2, &full[i], (kb0 + i) * BK, n0);
+          }
       }
+      auto mine = [&](long q) { return nprod == 1 || (q < pre ? pid == 0 : static_cast<int>(q & 1) == pid); };
       pdl_wait();
       pdl_trigger();
       for (int t = t_start; t < tiles && ok; t += t_stride) {
@@ -302,37 +313,34 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int m0 = m_tile(args, tq / nt, mt) * TM + rank * BM, n0 = (tq % nt) * bn;
         int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
         if (args.conv) conv_tile(args, m_tile(args, tq / nt, mt), cb0, cy0, cx0);
-        for (int kb = kb0; kb < kb1; ++kb) {
-          if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
-            ok = false;
-            break;
-          }
-          if constexpr (PAIR) {
-            const uint32_t full_lead = cluster_map(smem_addr(&full[stage]), 0);
-            if (leader) mbar_expect_tx(&full[stage], bytes);
-            tma_load_2d_pair(sA + stage * A_STAGE, &tmA, full_lead, kb * BK, m0);
-            tma_load_2d_pair(sB + stage * BSTG, &tmB, full_lead, kb * BK, n0 + rank * (bn / 2));
-            ++issued;
-            if (++stage == S) {
-              stage = 0;
-              phase ^= 1;
+        for (int kb = kb0; kb < kb1; ++kb, ++seq) {
+          if (mine(seq)) {
+            if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
+              ok = false;
+              break;
             }
-            continue;
+            if constexpr (PAIR) {
+              const uint32_t full_lead = cluster_map(smem_addr(&full[stage]), 0);
+              if (leader) mbar_expect_tx(&full[stage], bytes);
+              tma_load_2d_pair(sA + stage * A_STAGE, &tmA, full_lead, kb * BK, m0);
+              tma_load_2d_pair(sB + stage * BSTG, &tmB, full_lead, kb * BK, n0 + rank * (bn / 2));
+            } else {
+              const bool armed = seq < pre;  // this stage's weights were requested before the wait
+              if (!armed) mbar_expect_tx(&full[stage], bytes);
+              if (args.conv) {
+                const int tap = kb / args.cv_cgroups, cg = kb - tap * args.cv_cgroups;
+                const int ky = tap / args.cv_ks, kx = tap - ky * args.cv_ks;
+                tma_load_4d(sA + stage * A_STAGE, &tmA, &full[stage], cg * bke,
+                            cx0 * args.cv_stride - args.cv_pad + kx, cy0 * args.cv_stride - args.cv_pad + ky, cb0);
+              } else {
+                tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
+              }
+              if (!bres && !armed) tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * bke, n0);
+              if constexpr (NB == 2)
+                if (!armed) tma_load_2d(sB + stage * BSTG + BSTG / 2, &tmB2, &full[stage], kb * BK, n0);
+            }
+            last_mine = seq;
           }
-          const bool armed = issued < pre;  // this stage's weights were requested before the wait
-          if (!armed) mbar_expect_tx(&full[stage], bytes);
-          if (args.conv) {
-            const int tap = kb / args.cv_cgroups, cg = kb - tap * args.cv_cgroups;
-            const int ky = tap / args.cv_ks, kx = tap - ky * args.cv_ks;
-            tma_load_4d(sA + stage * A_STAGE, &tmA, &full[stage], cg * bke, cx0 * args.cv_stride - args.cv_pad + kx,
-                        cy0 * args.cv_stride - args.cv_pad + ky, cb0);
-          } else {
-            tma_load_2d(sA + stage * A_STAGE, &tmA, &full[stage], kb * BK, m0);
-          }
-          if (!bres && !armed) tma_load_2d(sB + stage * BSTG, &tmB, &full[stage], kb * bke, n0);
-          if constexpr (NB == 2)
-            if (!armed) tma_load_2d(sB + stage * BSTG + BSTG / 2, &tmB2, &full[stage], kb * BK, n0);
-          ++issued;
           if (++stage == S) {
             stage = 0;
             phase ^= 1;
@@ -340,17 +348,17 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
       }
       if (!ok) record_status(args.status, ELASTO_ERR_TIMEOUT);
-      // Drain: no copy may still be landing in shared memory when the CTA
-      // exits (returns at once on the normal path). In a pair only the even
-      // CTA's barriers see the copies; the cluster barrier before exit
-      // orders the odd CTA behind this drain.
-      for (int i = 0; i < S && i < issued && leader; ++i) {
-        if (stage == 0) {
-          stage = S;
-          phase ^= 1;
-        }
-        --stage;
-        PAIR ? mbar_wait_cluster(&full[stage], phase) : mbar_wait(&full[stage], phase);
+      // Drain: no copy this thread issued may still be landing in shared
+      // memory when the CTA exits (returns at once on the normal path): the
+      // stages of the sequence's last S k-blocks (no later k-block reuses
+      // them) that this thread issued. In a pair only the even CTA's
+      // barriers see the copies; the cluster barrier before exit orders the
+      // odd CTA behind this drain.
+      for (long q = seq - 1; leader && q >= 0 && q > seq - 1 - S; --q) {
+        if (!mine(q) || q > last_mine) continue;
+        const int st = static_cast<int>(q % S);
+        const uint32_t ph = static_cast<uint32_t>((q / S) & 1);
+        PAIR ? mbar_wait_cluster(&full[st], ph) : mbar_wait(&full[st], ph);
       }
       if (b_loaded) mbar_wait(bfull, 0);
     }
@@ -796,7 +804,8 @@ cudaError_t launch_epi(const GemmPlan& p, int M, cudaStream_t s) {
   } else {
     const int tiles = (a.conv ? conv_mtiles(a) : (M + BM - 1) / BM) * nt * (a.ksplit > 1 ? a.ksplit : 1);
     const int grid = tiles < num_sms() ? tiles : num_sms();
-    return launch_pdl(gemm_tc_kernel<EPI, NB, false>, dim3(grid), dim3(THREADS), SMEM_BYTES, s, p.tmA, p.tmB, p.tmB2,
+    return launch_pdl(gemm_tc_kernel<EPI, NB, false>, dim3(grid), dim3(a.conv ? THREADS_CONV : THREADS), SMEM_BYTES, s,
+                      p.tmA, p.tmB, p.tmB2,
                       p.tmC, p.tmR, a);
   }
 }
