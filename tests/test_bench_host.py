@@ -42,25 +42,29 @@ def test_clock_summary_idle_or_unparsable_samples():
 
 def test_committed_traffic_only_for_the_captured_source(tmp_path, monkeypatch):
     src = tmp_path / "kernel.cu"
+    hdr = tmp_path / "kernel.cuh"
     src.write_bytes(b"__global__ void k() {}\n")
-    sha = hashlib.sha256(src.read_bytes()).hexdigest()
+    hdr.write_bytes(b"#pragma once\n")
+    sha = hashlib.sha256(src.read_bytes() + hdr.read_bytes()).hexdigest()
+    assert bench.source_sha256([str(src), str(hdr)]) == sha
     prof = tmp_path / "profiles"
     prof.mkdir()
     (prof / "k.md").write_text("notes\n\ntraffic_kernel: k_kernel traffic_bytes_per_launch: 12.5e6 "
                                f"source_sha256: {sha}\n")
     (prof / "ignored.ncu-rep").write_text(f"traffic_kernel: k_kernel traffic_bytes_per_launch: 1 source_sha256: {sha}")
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.committed_traffic("k_kernel", str(src)) == 12.5e6
-    assert bench.committed_traffic("other_kernel", str(src)) is None
-    src.write_bytes(b"__global__ void k() { /* changed */ }\n")
-    assert bench.committed_traffic("k_kernel", str(src)) is None
+    files = [str(src), str(hdr)]
+    assert bench.committed_traffic("k_kernel", files) == 12.5e6
+    assert bench.committed_traffic("other_kernel", files) is None
+    hdr.write_bytes(b"#pragma once  // changed\n")  # any of the kernel's sources changing voids the figure
+    assert bench.committed_traffic("k_kernel", files) is None
 
 
 def test_committed_traffic_without_profiles(tmp_path, monkeypatch):
     src = tmp_path / "kernel.cu"
     src.write_bytes(b"x")
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench.committed_traffic("k_kernel", str(src)) is None
+    assert bench.committed_traffic("k_kernel", [str(src)]) is None
 
 
 def test_gemm_records_named_by_role():
