@@ -23,7 +23,7 @@
 //
 // Roles (320 threads):
 //   warp 0 lane 0  TMA producer: a unit's B (weight) k-blocks all at once into
-//                  the B region, A k-blocks through an 8-stage ring; attention
+//                  the B region, A k-blocks through a 7-stage ring; attention
 //                  Q, K, V into buffers that alias the ring. At the end of a
 //                  phase it already loads the B of its first unit of the next
 //                  GEMM phase.
@@ -35,14 +35,18 @@
 //                  PATCH work.
 // TMEM: GEMM accumulator in columns [0, bn); attention S in [0, n_pad), P (bf16
 // pairs) in [256, 256 + n_pad / 2), O in [384, 448).
-// Shared memory: [A ring 8 x 16 KB | B region 72 KB | barriers, exchange].
+// Shared memory: [A ring 7 x 16 KB | B region 72 KB | output staging 8 x 4 KB |
+// barriers, exchange, the current and next phase descriptors]. Outputs
+// (GEMM tiles, attention O) leave by TMA stores of 32-row boxes staged per
+// warp (128-byte rows in the 128-byte swizzle).
 //
-// Memory ordering across phases: results are written with ordinary stores;
-// every thread fences its global writes against the async proxy (TMA reads of
-// them in the next phase), the CTA synchronises, one thread releases its
-// arrival and acquires everyone's; the TMA issuer fences again before its
-// first load of the phase. Data written inside the kernel is never read
-// through the non-coherent cache.
+// Memory ordering across phases: a phase's results are written by TMA stores
+// (waited for until complete before the barrier) or ordinary stores; every
+// thread fences against the async proxy (the TMA reads and writes on either
+// side), the CTA synchronises, one thread releases its arrival and acquires
+// everyone's; the TMA issuer fences again before its first load of the
+// phase. Data written inside the kernel is never read through the
+// non-coherent cache.
 //
 // Every wait (mbarrier or grid counter) is bounded; one that gives up records
 // ELASTO_ERR_TIMEOUT in the status word and raises an abort flag that every
