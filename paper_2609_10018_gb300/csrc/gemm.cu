@@ -312,7 +312,14 @@ __global__ void __launch_bounds__(THREADS_CONV, 1)
         const int kb0 = kSplit ? (t / mn_tiles) * nk / ks : 0, kb1 = kSplit ? (t / mn_tiles + 1) * nk / ks : nk;
         const int m0 = m_tile(args, tq / nt, mt) * TM + rank * BM, n0 = (tq % nt) * bn;
         int cb0 = 0, cy0 = 0, cx0 = 0;  // implicit conv: first image, output row and column of the tile
-        if (args.conv) conv_tile(args, m_tile(args, tq / nt, mt), cb0, cy0, cx0);
+        int cg = 0, kx = 0, ky = 0;     // implicit conv: the k-block's channel group and tap, advanced in step
+        if (args.conv) {
+          conv_tile(args, m_tile(args, tq / nt, mt), cb0, cy0, cx0);
+          const int tap = kb0 / args.cv_cgroups;
+          cg = kb0 - tap * args.cv_cgroups;
+          ky = tap / args.cv_ks;
+          kx = tap - ky * args.cv_ks;
+        }
         for (int kb = kb0; kb < kb1; ++kb, ++seq) {
           if (mine(seq)) {
             if (!(PAIR ? mbar_wait_cluster(&empty[stage], phase ^ 1) : mbar_wait(&empty[stage], phase ^ 1))) {
@@ -328,8 +335,6 @@ __global__ void __launch_bounds__(THREADS_CONV, 1)
               const bool armed = seq < pre;  // this stage's weights were requested before the wait
               if (!armed) mbar_expect_tx(&full[stage], bytes);
               if (args.conv) {
-                const int tap = kb / args.cv_cgroups, cg = kb - tap * args.cv_cgroups;
-                const int ky = tap / args.cv_ks, kx = tap - ky * args.cv_ks;
                 tma_load_4d(sA + stage * A_STAGE, &tmA, &full[stage], cg * bke,
                             cx0 * args.cv_stride - args.cv_pad + kx, cy0 * args.cv_stride - args.cv_pad + ky, cb0);
               } else {
@@ -344,6 +349,13 @@ __global__ void __launch_bounds__(THREADS_CONV, 1)
           if (++stage == S) {
             stage = 0;
             phase ^= 1;
+          }
+          if (++cg == args.cv_cgroups) {  // (meaningful for convolutions only)
+            cg = 0;
+            if (++kx == args.cv_ks) {
+              kx = 0;
+              ++ky;
+            }
           }
         }
       }
@@ -399,18 +411,20 @@ __global__ void __launch_bounds__(THREADS_CONV, 1)
             // 8-row groups 256 bytes apart
             if constexpr (!PAIR && NB == 1)
               tc_mma(dtm, sdesc_sw32(a0, 16, 256), sdesc_sw32(b0, 16, 256), idesc, kb != kb0);
-          } else
+          } else {
+            // the stage's descriptors once; a K = 16 step is +32 bytes = +2 in
+            // the start-address field (the tiles are 1024-byte aligned, so it
+            // never carries out of the field)
+            const uint64_t da = sdesc_sw128(a0, 16, 1024), db = sdesc_sw128(b0, 16, 1024);
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k) {
-            if constexpr (PAIR) {
-              tc_mma_pair(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
-                          kb != kb0 || k != 0);
-            } else {
-              tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + k * 32, 16, 1024), idesc,
-                     kb != kb0 || k != 0);
-              if constexpr (NB == 2)  // low half of the weights: acc += A . W_lo^T
-                tc_mma(dtm, sdesc_sw128(a0 + k * 32, 16, 1024), sdesc_sw128(b0 + BSTG / 2 + k * 32, 16, 1024),
-                       idesc, 1u);
+            for (int k = 0; k < BK / 16; ++k) {
+              if constexpr (PAIR) {
+                tc_mma_pair(dtm, da + 2 * k, db + 2 * k, idesc, kb != kb0 || k != 0);
+              } else {
+                tc_mma(dtm, da + 2 * k, db + 2 * k, idesc, kb != kb0 || k != 0);
+                if constexpr (NB == 2)  // low half of the weights: acc += A . W_lo^T
+                  tc_mma(dtm, da + 2 * k, sdesc_sw128(b0 + BSTG / 2, 16, 1024) + 2 * k, idesc, 1u);
+              }
             }
           }
           issued = true;
